@@ -1,0 +1,387 @@
+"""Benchmark of the HDL hot path on GB300: one step = re-scoring of every root
+token under both contexts (fused LM-head GEMM + log-sum-exp + gather, and the
+divergence), top-k branch selection, continuation allocation and suffix-only
+masks, over one synthetic workload resident in HBM.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--workload code]
+    python bench.py --impl reference ...   # the fp64 CPU oracle, timed
+
+Prints one JSON line.  ``value`` = root tokens per second (each token scored
+under both contexts) over all ranks; ``e2e`` = the same with the per-step
+host->device copy of the inputs and device->host copy of the results.
+Multi-GPU runs (torchrun) give every rank its own independent workload
+(weak scaling, no collective on the data path).
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import subprocess
+import sys
+import time
+
+os.environ.setdefault("OPENBLAS_NUM_THREADS", str(os.cpu_count() or 1))
+
+import numpy as np  # noqa: E402
+import torch  # noqa: E402
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import hdl_synth  # noqa: E402
+
+METRIC = "re-scored tokens/sec (both contexts) and % of GB300 bf16 dense tensor peak"
+L2_BYTES = 129 * 1024 * 1024
+
+
+def parse():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=10)
+    p.add_argument("--warmup", type=int, default=3)
+    p.add_argument("--workload", default="code",
+                   help="tiny | math | code | agent | sweep_V<vocab>_N<tokens>")
+    p.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
+    p.add_argument("--no-e2e", action="store_true")
+    p.add_argument("--no-cpu", action="store_true")
+    p.add_argument("--cpu-seconds", type=float, default=12.0)
+    return p.parse_args()
+
+
+def spec_for(name: str, seed: int) -> hdl_synth.Spec:
+    import dataclasses
+    if name in hdl_synth.SPECS:
+        return dataclasses.replace(hdl_synth.SPECS[name], seed=seed)
+    if name.startswith("sweep_V"):
+        v, n = name[len("sweep_V"):].split("_N")
+        return hdl_synth.sweep_spec(int(v), int(n), seed=seed)
+    raise SystemExit(f"unknown workload {name}")
+
+
+def peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        mp = json.load(open(path))
+        return (mp["bf16_tflops"], mp["bf16_tflops_sustained"], mp["hbm_gbs"], "measured")
+    return 1900.0, 1700.0, 6800.0, "fallback"
+
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons sampled during the timed region."""
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.Q}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            out, _ = self.proc.communicate(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+            out, _ = self.proc.communicate()
+        sm, smax, power, reasons = [], None, [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in out.splitlines():
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                smax = float(f[2])
+                power.append(float(f[3]))
+            except ValueError:
+                continue
+            for name, val in zip(names, f[5:9]):
+                if val.lower().startswith("active"):
+                    reasons.add(name)
+        return {"sm_mhz": float(np.median(sm)) if sm else None, "sm_max_mhz": smax,
+                "power_w_max": max(power) if power else None, "samples": len(sm),
+                "reasons": sorted(reasons)}
+
+
+class Path:
+    """Device buffers and the four library calls of one step."""
+
+    def __init__(self, hdl, wl):
+        self.hdl, self.wl = hdl, wl
+        dev = wl.h_orig.device
+        N, R, k = wl.n_tokens, wl.n_roots, wl.spec.k
+        self.C = wl.cont_offsets.numel() - 1
+        self.lp0 = torch.empty(N, dtype=torch.float32, device=dev)
+        self.lp1 = torch.empty_like(self.lp0)
+        self.delta = torch.empty_like(self.lp0)
+        need = hdl.hdl_rescore_workspace_bytes(N, wl.spec.d, wl.spec.vocab, wl.h_orig.dtype)
+        self.ws = torch.empty(need, dtype=torch.uint8, device=dev)
+        self.bp = torch.empty((R, k), dtype=torch.int32, device=dev)
+        self.ns = torch.empty(R, dtype=torch.int32, device=dev)
+        self.bd = torch.empty((R, k), dtype=torch.float32, device=dev)
+        self.cb = torch.empty(self.C, dtype=torch.int32, device=dev)
+        self.mask = torch.zeros(wl.cont_valid.numel(), dtype=torch.uint8, device=dev)
+
+    def rescore(self, stream):
+        w = self.wl
+        self.hdl.hdl_rescore(w.h_orig, w.h_hind, w.w, w.targets, self.lp0, self.lp1,
+                             self.delta, self.ws, stream=stream)
+
+    def downstream(self, stream):
+        w, h = self.wl, self.hdl
+        h.hdl_select_branches(self.delta, w.valid, w.root_offsets, w.spec.k,
+                              branch_pos=self.bp, n_selected=self.ns, branch_delta=self.bd,
+                              stream=stream)
+        h.hdl_assign_continuations(self.ns, self.bp, w.conts_per_root, cont_branch=self.cb,
+                                   stream=stream)
+        h.hdl_suffix_mask(self.cb, w.cont_offsets, w.cont_valid, mask=self.mask, stream=stream)
+
+    LAUNCHES_PER_STEP = 5  # rescore (fused GEMM + LSE), merge, select, assign, mask
+
+
+def dist_setup():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch.distributed as dist
+        backend = "nccl" if torch.cuda.is_available() else "gloo"
+        if torch.cuda.is_available():
+            torch.cuda.set_device(local)
+        dist.init_process_group(backend)
+    elif torch.cuda.is_available():
+        torch.cuda.set_device(local)
+    return world, rank, local
+
+
+def barrier(world):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def max_over_ranks(x: float, world: int) -> float:
+    if world == 1:
+        return x
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64,
+                     device="cuda" if torch.cuda.is_available() else "cpu")
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def cpu_oracle_sample(wl, seconds: float, rng_seed: int = 0):
+    """Time the fp64 oracle on sampled tokens of the workload: log-probs of
+    both contexts for a growing sample until ``seconds`` of CPU work, plus
+    selection / allocation / masks over the whole workload (on its scores)."""
+    import oracle
+
+    def to_f64(t):  # exact widening of the bf16 / fp32 inputs
+        t = t.detach().cpu().contiguous()
+        if t.dtype == torch.bfloat16:
+            return oracle.widen(t.view(torch.int16).numpy(), "bf16")
+        return oracle.widen(t.numpy(), "f32")
+    N = wl.n_tokens
+    W = to_f64(wl.w)
+    y_all = wl.targets.cpu().numpy()
+    rng = np.random.default_rng(rng_seed)
+    done, t_lp, block = 0, 0.0, 8
+    delta_s = []
+    while t_lp < seconds and done < N:
+        rows = np.sort(rng.choice(N, size=min(block, N - done), replace=False))
+        idx = torch.from_numpy(rows).to(wl.h_orig.device)
+        h0 = to_f64(wl.h_orig.index_select(0, idx))
+        h1 = to_f64(wl.h_hind.index_select(0, idx))
+        t0 = time.perf_counter()
+        lp0 = oracle.target_logprobs(h0, W, y_all[rows])
+        lp1 = oracle.target_logprobs(h1, W, y_all[rows])
+        delta_s.append(oracle.hindsight_divergence(lp1, lp0))
+        t_lp += time.perf_counter() - t0
+        done += len(rows)
+        block = min(block * 2, 256)
+    del W
+    # downstream steps over the full workload, on scores of its shape
+    offs = wl.root_offsets.cpu().numpy()
+    valid = wl.valid.cpu().numpy()
+    delta = np.abs(np.random.default_rng(1).normal(size=N))
+    t0 = time.perf_counter()
+    pos, nsel, _ = oracle.select_branches(delta, valid, offs, wl.spec.k)
+    cb = oracle.assign_continuations(nsel, pos, wl.conts_per_root.cpu().numpy())
+    oracle.suffix_mask(cb, wl.cont_offsets.cpu().numpy(), wl.cont_valid.cpu().numpy())
+    t_down = time.perf_counter() - t0
+    per_token = t_lp / done + t_down / N
+    return {"value": 1.0 / per_token, "unit": "root tokens/s",
+            "cores": int(os.environ.get("OPENBLAS_NUM_THREADS", os.cpu_count() or 1)),
+            "kind": "oracle",
+            "sample": (f"log-probs of both contexts for {done} random tokens of {N} "
+                       f"({t_lp:.1f} s), selection + allocation + masks over all {N} "
+                       f"tokens ({t_down:.2f} s); per-token times added")}
+
+
+def run_reference(args, world, rank):
+    if rank != 0:
+        return
+    spec = spec_for(args.workload, seed=0)
+    dev = "cuda" if torch.cuda.is_available() else "cpu"
+    wl = hdl_synth.generate(spec, device=dev)
+    per_step = max(1.0, min(args.cpu_seconds, 150.0 / max(1, args.steps + args.warmup)))
+    for _ in range(args.warmup):
+        cpu_oracle_sample(wl, per_step / 4)
+    vals, cb = [], None
+    t0 = time.perf_counter()
+    for i in range(args.steps):
+        cb = cpu_oracle_sample(wl, per_step, rng_seed=i)
+        vals.append(cb["value"])
+    wall = time.perf_counter() - t0
+    value = float(np.mean(vals))
+    cb["value"] = value
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "root tokens/s",
+            "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": 1e3 * wall / max(1, args.steps), "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": spec.name, "n_tokens": wl.n_tokens, "d": spec.d,
+                       "vocab": spec.vocab, "roots": spec.n_roots, "k": spec.k},
+            "cpu_baseline": cb,
+            "e2e": {"value": value, "unit": "root tokens/s", "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def run_gpu(args, world, rank, local):
+    import paper_2609_36864_gb300 as hdl
+    from paper_2609_36864_gb300 import build as b
+    if rank == 0 or not b.up_to_date():
+        b.build()
+    barrier(world)
+    spec = spec_for(args.workload, seed=rank)
+    dev = torch.device("cuda", local)
+    wl = hdl_synth.generate(spec, device=dev)
+    torch.cuda.synchronize()
+    path = Path(hdl, wl)
+    stream = torch.cuda.current_stream()
+    N, d, V = wl.n_tokens, spec.d, spec.vocab
+    flops = 2.0 * (2 * N) * d * V
+    in_bytes = sum(t.numel() * t.element_size() for t in (wl.h_orig, wl.h_hind, wl.w))
+
+    for _ in range(max(args.warmup, 3)):
+        path.rescore(stream)
+        path.downstream(stream)
+    code, raw = hdl.hdl_device_status(path.ws, stream)
+    assert code == hdl.HDL_OK, (code, raw)
+
+    # ---- kernel-only: inputs resident in HBM, larger than L2
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(args.steps)]
+    clocks = ClockSampler(local)
+    barrier(world)
+    torch.cuda.synchronize()
+    clocks.start()
+    t_start = torch.cuda.Event(enable_timing=True)
+    t_end = torch.cuda.Event(enable_timing=True)
+    t_start.record(stream)
+    for i in range(args.steps):
+        ev[i][0].record(stream)
+        path.rescore(stream)
+        ev[i][1].record(stream)
+        path.downstream(stream)
+    t_end.record(stream)
+    torch.cuda.synchronize()
+    clk = clocks.stop()
+    barrier(world)
+    code, raw = hdl.hdl_device_status(path.ws, stream)
+    assert code == hdl.HDL_OK, (code, raw)
+    total_ms = max_over_ranks(t_start.elapsed_time(t_end), world)
+    rescore_ms = float(np.mean([a.elapsed_time(b_) for a, b_ in ev]))
+    value = world * N * args.steps / (total_ms / 1e3)
+
+    # ---- end to end: host inputs copied in, results copied out, every step
+    e2e = None
+    if not args.no_e2e:
+        host_in = {k: getattr(wl, k).cpu().pin_memory() for k in
+                   ("h_orig", "h_hind", "targets", "valid", "root_offsets", "conts_per_root",
+                    "cont_offsets", "cont_valid")}
+        outs = (path.bp, path.ns, path.bd, path.mask)
+        host_out = [torch.empty(t.shape, dtype=t.dtype, pin_memory=True) for t in outs]
+        h2d = sum(t.numel() * t.element_size() for t in host_in.values())
+        d2h = sum(t.numel() * t.element_size() for t in host_out)
+
+        def e2e_step():
+            for k_, t in host_in.items():
+                getattr(wl, k_).copy_(t, non_blocking=True)
+            path.rescore(stream)
+            path.downstream(stream)
+            for hst, dv in zip(host_out, outs):
+                hst.copy_(dv, non_blocking=True)
+
+        for _ in range(2):
+            e2e_step()
+        torch.cuda.synchronize()
+        barrier(world)
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(args.steps):
+            e2e_step()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        e2e_ms = max_over_ranks(e0.elapsed_time(e1), world)
+        e2e = {"value": world * N * args.steps / (e2e_ms / 1e3), "unit": "root tokens/s",
+               "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h}
+
+    cpu = None
+    if rank == 0 and not args.no_cpu:
+        cpu = cpu_oracle_sample(wl, args.cpu_seconds)
+
+    if rank != 0:
+        return
+    burst, sustained, hbm, src = peaks()
+    achieved = flops / (rescore_ms / 1e3) / 1e12
+    line = {
+        "metric": METRIC, "value": value, "unit": "root tokens/s", "n_gpus": world,
+        "steps": args.steps, "warmup": max(args.warmup, 3),
+        "ms_per_step": total_ms / args.steps, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16" if spec.dtype == "bf16" else "f32",
+        "data": "synthetic",
+        "config": {"workload": spec.name, "n_tokens": N, "d": d, "vocab": V,
+                   "roots": spec.n_roots, "k": spec.k, "conts": path.C,
+                   "context_rows_per_step": 2 * N,
+                   "l2": f"inputs larger than L2 ({in_bytes / 2**30:.2f} GiB resident)"},
+        "tflops": flops * args.steps / (total_ms / 1e3) / 1e12,
+        "pct_bf16_peak": 100.0 * (flops * args.steps / (total_ms / 1e3) / 1e12) / burst,
+        "roofline": {"bound": "tensor", "kernel": "rescore_lse_kernel (+ merge)",
+                     "achieved": achieved, "peak": sustained, "unit": "TFLOP/s",
+                     "frac": achieved / sustained, "peak_kind": f"bf16 sustained ({src})",
+                     "frac_of_burst": achieved / burst, "traffic": None,
+                     "rescore_ms": rescore_ms},
+        "cpu_baseline": cpu, "e2e": e2e, "clocks": clk,
+        "gpu_launches": Path.LAUNCHES_PER_STEP * args.steps,
+    }
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    args = parse()
+    world, rank, local = dist_setup()
+    if args.impl == "reference":
+        run_reference(args, world, rank)
+    else:
+        run_gpu(args, world, rank, local)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,257 @@
+"""Python binding of libhdl, the GB300 kernels for HDL (arXiv 2609.36864).
+
+Each function has the name of the C entry point it calls (include/hdl.h) and
+only marshals arguments: it checks devices, dtypes and contiguity, fills in
+the current CUDA stream, optionally allocates output tensors with torch, and
+passes raw pointers.  Every step of the computation runs in the library's
+CUDA kernels; there is no CPU fallback.  Importing this package does not load
+the library; the first call does, and fails loudly if libhdl.so is missing.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+from typing import Optional
+
+import torch
+
+__all__ = [
+    "HdlError", "lib", "library_path", "HDL_OK", "HDL_BF16", "HDL_F32",
+    "hdl_abi_version", "hdl_status_string", "hdl_rescore_workspace_bytes",
+    "hdl_rescore", "hdl_device_status", "hdl_select_branches",
+    "hdl_assign_continuations", "hdl_suffix_mask",
+]
+
+HDL_OK, HDL_ERR_INVALID_ARG, HDL_ERR_UNSUPPORTED, HDL_ERR_WORKSPACE = 0, 1, 2, 3
+HDL_ERR_CUDA, HDL_ERR_TIMEOUT, HDL_ERR_BAD_TARGET = 4, 5, 6
+HDL_BF16, HDL_F32 = 0, 1
+
+_PKG = os.path.dirname(os.path.abspath(__file__))
+_lib = None
+_lock = threading.Lock()
+
+
+def library_path() -> str:
+    return os.path.join(_PKG, "libhdl.so")
+
+
+class HdlError(RuntimeError):
+    def __init__(self, fn: str, code: int):
+        self.code = code
+        super().__init__(f"{fn} failed: {_status_name(code)} ({code})")
+
+
+class _SelectOpts(ctypes.Structure):
+    _fields_ = [("min_gap", ctypes.c_int32), ("gap_mode", ctypes.c_int32),
+                ("lo", ctypes.c_int32), ("hi", ctypes.c_int32)]
+
+
+def _declare(L):
+    vp, i32, i64, sz = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.c_size_t
+    L.hdl_abi_version.restype = i32
+    L.hdl_abi_version.argtypes = []
+    L.hdl_status_string.restype = ctypes.c_char_p
+    L.hdl_status_string.argtypes = [ctypes.c_int]
+    L.hdl_rescore_workspace_bytes.restype = sz
+    L.hdl_rescore_workspace_bytes.argtypes = [i64, i32, i32, ctypes.c_int]
+    L.hdl_rescore.restype = ctypes.c_int
+    L.hdl_rescore.argtypes = [vp, vp, vp, ctypes.c_int, vp, i64, i32, i32, vp, vp, vp,
+                              vp, sz, vp]
+    L.hdl_device_status.restype = ctypes.c_int
+    L.hdl_device_status.argtypes = [vp, sz, vp, ctypes.POINTER(ctypes.c_uint32)]
+    L.hdl_select_branches.restype = ctypes.c_int
+    L.hdl_select_branches.argtypes = [vp, vp, i64, vp, i32, i32,
+                                      ctypes.POINTER(_SelectOpts), vp, vp, vp, vp]
+    L.hdl_assign_continuations.restype = ctypes.c_int
+    L.hdl_assign_continuations.argtypes = [vp, vp, i32, i32, vp, i32, vp, i64, vp]
+    L.hdl_suffix_mask.restype = ctypes.c_int
+    L.hdl_suffix_mask.argtypes = [vp, vp, i32, vp, vp, i64, vp]
+    return L
+
+
+def lib():
+    """Load libhdl.so (built by ``__graft_entry__.build()``); raise if absent."""
+    global _lib
+    if _lib is None:
+        with _lock:
+            if _lib is None:
+                path = library_path()
+                if not os.path.exists(path):
+                    raise RuntimeError(
+                        f"libhdl.so not found at {path}: build it first with "
+                        "`python -c 'import __graft_entry__ as g; g.build()'`")
+                _lib = _declare(ctypes.CDLL(path))
+    return _lib
+
+
+def _status_name(code: int) -> str:
+    try:
+        return lib().hdl_status_string(code).decode()
+    except Exception:  # the name is only cosmetic
+        return str(code)
+
+
+def _check(fn: str, code: int):
+    if code != HDL_OK:
+        raise HdlError(fn, code)
+
+
+def _ptr(t: Optional[torch.Tensor]):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream) -> ctypes.c_void_p:
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    if isinstance(stream, torch.cuda.Stream):
+        return ctypes.c_void_p(stream.cuda_stream)
+    return ctypes.c_void_p(int(stream))
+
+
+def _dev(t: torch.Tensor, name: str, dtype=None):
+    if not isinstance(t, torch.Tensor):
+        raise TypeError(f"{name} must be a torch.Tensor")
+    if t.device.type != "cuda":
+        raise ValueError(f"{name} must be a CUDA tensor (got {t.device})")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    if dtype is not None and t.dtype != dtype:
+        raise ValueError(f"{name} must be {dtype} (got {t.dtype})")
+
+
+def _hdl_dtype(t: torch.Tensor) -> int:
+    if t.dtype == torch.bfloat16:
+        return HDL_BF16
+    if t.dtype == torch.float32:
+        return HDL_F32
+    raise ValueError(f"hidden states / LM head must be bf16 or fp32 (got {t.dtype})")
+
+
+# -------------------------------------------------------------- entry points
+def hdl_abi_version() -> int:
+    return int(lib().hdl_abi_version())
+
+
+def hdl_status_string(code: int) -> str:
+    return lib().hdl_status_string(code).decode()
+
+
+def hdl_rescore_workspace_bytes(n_tokens: int, d: int, vocab: int, dtype=HDL_BF16) -> int:
+    if isinstance(dtype, torch.dtype):
+        dtype = HDL_BF16 if dtype == torch.bfloat16 else HDL_F32
+    return int(lib().hdl_rescore_workspace_bytes(n_tokens, d, vocab, dtype))
+
+
+def hdl_rescore(h_orig, h_hind, w_lmhead, targets, logp_orig=None, logp_hind=None,
+                delta=None, workspace=None, want_delta=True, stream=None):
+    """log p^0(y_t), log p^H(y_t) and |Delta_t| for every token (Eq. div).
+
+    Returns (logp_orig, logp_hind, delta, workspace); outputs not given are
+    allocated.  Asynchronous on ``stream``; device-side errors surface through
+    :func:`hdl_device_status` on the returned workspace.
+    """
+    for t, n in ((h_orig, "h_orig"), (h_hind, "h_hind"), (w_lmhead, "w_lmhead")):
+        _dev(t, n)
+    _dev(targets, "targets", torch.int32)
+    dt = _hdl_dtype(h_orig)
+    if h_hind.dtype != h_orig.dtype or w_lmhead.dtype != h_orig.dtype:
+        raise ValueError("h_orig, h_hind and w_lmhead must share one dtype")
+    N, d = h_orig.shape
+    V = w_lmhead.shape[0]
+    if h_hind.shape != (N, d) or w_lmhead.shape != (V, d) or targets.shape != (N,):
+        raise ValueError("shape mismatch between h_orig, h_hind, w_lmhead, targets")
+    dev = h_orig.device
+    if logp_orig is None:
+        logp_orig = torch.empty(N, dtype=torch.float32, device=dev)
+    if logp_hind is None:
+        logp_hind = torch.empty(N, dtype=torch.float32, device=dev)
+    if delta is None and want_delta:
+        delta = torch.empty(N, dtype=torch.float32, device=dev)
+    for t, n in ((logp_orig, "logp_orig"), (logp_hind, "logp_hind")):
+        _dev(t, n, torch.float32)
+    if delta is not None:
+        _dev(delta, "delta", torch.float32)
+    need = hdl_rescore_workspace_bytes(N, d, V, dt)
+    if workspace is None:
+        workspace = torch.empty(max(need, 256), dtype=torch.uint8, device=dev)
+    _dev(workspace, "workspace", torch.uint8)
+    code = lib().hdl_rescore(_ptr(h_orig), _ptr(h_hind), _ptr(w_lmhead), dt, _ptr(targets),
+                             N, d, V, _ptr(logp_orig), _ptr(logp_hind), _ptr(delta),
+                             _ptr(workspace), workspace.numel(), _stream(stream))
+    _check("hdl_rescore", code)
+    return logp_orig, logp_hind, delta, workspace
+
+
+def hdl_device_status(workspace: torch.Tensor, stream=None):
+    """(status code, raw status word) of a re-scoring workspace; synchronises."""
+    raw = ctypes.c_uint32(0)
+    code = lib().hdl_device_status(_ptr(workspace), workspace.numel(), _stream(stream),
+                                   ctypes.byref(raw))
+    return int(code), int(raw.value)
+
+
+def hdl_select_branches(delta, valid, root_offsets, k: int, min_gap: int = 0,
+                        gap_mode: int = 0, lo: int = 0, hi: int = 0, branch_pos=None,
+                        n_selected=None, branch_delta=None, want_delta=True, stream=None):
+    """Top-k branch points per root; returns (branch_pos [R,k], n_selected [R], branch_delta)."""
+    _dev(delta, "delta", torch.float32)
+    if valid is not None:
+        _dev(valid, "valid", torch.uint8)
+    _dev(root_offsets, "root_offsets", torch.int64)
+    R = root_offsets.numel() - 1
+    dev = delta.device
+    if branch_pos is None:
+        branch_pos = torch.empty((R, k), dtype=torch.int32, device=dev)
+    if n_selected is None:
+        n_selected = torch.empty(R, dtype=torch.int32, device=dev)
+    if branch_delta is None and want_delta:
+        branch_delta = torch.empty((R, k), dtype=torch.float32, device=dev)
+    opts = _SelectOpts(min_gap, gap_mode, lo, hi)
+    code = lib().hdl_select_branches(_ptr(delta), _ptr(valid), delta.numel(),
+                                     _ptr(root_offsets), R, k, ctypes.byref(opts),
+                                     _ptr(branch_pos), _ptr(n_selected), _ptr(branch_delta),
+                                     _stream(stream))
+    _check("hdl_select_branches", code)
+    return branch_pos, n_selected, branch_delta
+
+
+def hdl_assign_continuations(n_selected, branch_pos, conts_per_root, extra_to_higher=True,
+                             cont_branch=None, n_cont: Optional[int] = None, stream=None):
+    """Root-relative branch position of every continuation (root-major)."""
+    _dev(n_selected, "n_selected", torch.int32)
+    _dev(branch_pos, "branch_pos", torch.int32)
+    _dev(conts_per_root, "conts_per_root", torch.int32)
+    R, k = branch_pos.shape
+    if cont_branch is None:
+        if n_cont is None:
+            raise ValueError("give cont_branch or n_cont (the total continuation count)")
+        cont_branch = torch.empty(n_cont, dtype=torch.int32, device=branch_pos.device)
+    _dev(cont_branch, "cont_branch", torch.int32)
+    code = lib().hdl_assign_continuations(_ptr(n_selected), _ptr(branch_pos), R, k,
+                                          _ptr(conts_per_root), 1 if extra_to_higher else 0,
+                                          _ptr(cont_branch), cont_branch.numel(),
+                                          _stream(stream))
+    _check("hdl_assign_continuations", code)
+    return cont_branch
+
+
+def hdl_suffix_mask(cont_branch, cont_offsets, cont_valid=None, mask=None,
+                    mask_len: Optional[int] = None, stream=None):
+    """Suffix-only loss mask of packed continuations (uint8)."""
+    _dev(cont_branch, "cont_branch", torch.int32)
+    _dev(cont_offsets, "cont_offsets", torch.int64)
+    if cont_valid is not None:
+        _dev(cont_valid, "cont_valid", torch.uint8)
+    C = cont_branch.numel()
+    if mask is None:
+        if mask_len is None:
+            mask_len = cont_valid.numel() if cont_valid is not None else None
+        if mask_len is None:
+            raise ValueError("give mask, mask_len or cont_valid")
+        mask = torch.zeros(mask_len, dtype=torch.uint8, device=cont_branch.device)
+    _dev(mask, "mask", torch.uint8)
+    code = lib().hdl_suffix_mask(_ptr(cont_branch), _ptr(cont_offsets), C, _ptr(cont_valid),
+                                 _ptr(mask), mask.numel(), _stream(stream))
+    _check("hdl_suffix_mask", code)
+    return mask

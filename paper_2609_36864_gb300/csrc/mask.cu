@@ -1,0 +1,196 @@
+// Continuation allocation (Section 4.1 "Rollout protocols", Table
+// fork-ablation, Section 4.4) and suffix-only loss masks (Section 3.3,
+// Eq. branch-sampling).
+#include <cuda_runtime.h>
+
+#include <cstdint>
+
+#include "hdl.h"
+#include "hdl_internal.h"
+
+namespace hdl {
+namespace {
+
+constexpr int kAssignThreads = 1024;
+constexpr int kMaskThreads = 256;
+
+// Rank of the branch point that continuation j (of C) of a root with n
+// points branches from: point i gets floor(C/n) + [i < C mod n] consecutive
+// continuations (extra to the higher-ranked points), or
+// floor(C/n) + [i >= n - C mod n] (extra to the lower-ranked ones).
+__device__ __forceinline__ int cont_rank(int j, int C, int n, bool extra_to_higher) {
+  const int base = C / n, rem = C % n;
+  if (extra_to_higher) {
+    const int head = rem * (base + 1);
+    return j < head ? j / (base + 1) : rem + (j - head) / base;
+  }
+  const int head = (n - rem) * base;
+  return j < head ? j / base : (n - rem) + (j - head) / (base + 1);
+}
+
+// One CTA: an exclusive scan of the continuation counts gives each root's
+// first output slot; each thread then fills its root's continuations.
+__global__ void __launch_bounds__(kAssignThreads)
+    assign_continuations_kernel(const int32_t* __restrict__ n_selected,
+                                const int32_t* __restrict__ branch_pos, int32_t n_roots,
+                                int32_t k, const int32_t* __restrict__ conts_per_root,
+                                int32_t extra_to_higher, int32_t* __restrict__ cont_branch,
+                                int64_t capacity) {
+  __shared__ int64_t warp_sums[kAssignThreads / 32];
+  __shared__ int64_t carry;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) carry = 0;
+  __syncthreads();
+  for (int base = 0; base < n_roots; base += kAssignThreads) {
+    const int r = base + threadIdx.x;
+    int64_t C = 0;
+    if (r < n_roots) {
+      const int32_t c = conts_per_root[r];
+      C = c > 0 ? c : 0;
+    }
+    // inclusive warp scan, then across warps
+    int64_t v = C;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int64_t u = __shfl_up_sync(0xffffffffu, v, o);
+      if (lane >= o) v += u;
+    }
+    if (lane == 31) warp_sums[warp] = v;
+    __syncthreads();
+    if (warp == 0) {
+      int64_t w = warp_sums[lane];
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int64_t u = __shfl_up_sync(0xffffffffu, w, o);
+        if (lane >= o) w += u;
+      }
+      warp_sums[lane] = w;
+    }
+    __syncthreads();
+    const int64_t first = carry + (warp > 0 ? warp_sums[warp - 1] : 0) + (v - C);
+    if (r < n_roots && C > 0) {
+      int n = n_selected[r];
+      n = n < 0 ? 0 : (n > k ? k : n);
+      for (int j = 0; j < static_cast<int>(C); ++j) {
+        const int64_t o = first + j;
+        if (o >= capacity) break;
+        cont_branch[o] =
+            n == 0 ? -1
+                   : branch_pos[static_cast<int64_t>(r) * k +
+                                cont_rank(j, static_cast<int>(C), n, extra_to_higher != 0)];
+      }
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) carry += warp_sums[kAssignThreads / 32 - 1];
+    __syncthreads();
+  }
+}
+
+// Index of the continuation holding mask byte p: the last c with
+// offs[c] <= p, searched in [0, n).
+__device__ __forceinline__ int find_cont(const int64_t* offs, int n, int64_t p) {
+  int lo = 0, hi = n - 1;
+  while (lo < hi) {
+    const int mid = (lo + hi + 1) >> 1;
+    if (offs[mid] <= p) lo = mid; else hi = mid - 1;
+  }
+  return lo;
+}
+
+// mask byte of continuation c at absolute position p
+__device__ __forceinline__ uint8_t mask_byte(const int32_t* cb, const int64_t* offs, int c,
+                                             int64_t p, const uint8_t* valid) {
+  const int32_t b = cb[c];
+  const int64_t t = p - offs[c];
+  const bool on = b >= 0 && t >= b && (valid == nullptr || valid[p] != 0);
+  return on ? 1 : 0;
+}
+
+// Grid-stride over 16-byte chunks of [lo, hi): whole chunks are read and
+// written with 16-byte vector accesses, the two edge chunks byte by byte.
+template <bool kVec>
+__global__ void __launch_bounds__(kMaskThreads)
+    suffix_mask_kernel(const int32_t* __restrict__ cb, const int64_t* __restrict__ offs,
+                       int32_t n_cont, const uint8_t* __restrict__ valid,
+                       uint8_t* __restrict__ mask, int64_t mask_len) {
+  int64_t lo = offs[0], hi = offs[n_cont];
+  lo = lo < 0 ? 0 : lo;
+  hi = hi > mask_len ? mask_len : hi;
+  if (hi <= lo) return;
+  const int64_t c0 = lo / 16, c1 = (hi + 15) / 16;
+  for (int64_t ch = c0 + blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; ch < c1;
+       ch += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+    const int64_t p0 = ch * 16;
+    const int64_t first = p0 > lo ? p0 : lo;
+    int c = find_cont(offs, n_cont, first);
+    if (kVec && p0 >= lo && p0 + 16 <= hi) {
+      uint4 vv = make_uint4(0xFFFFFFFFu, 0xFFFFFFFFu, 0xFFFFFFFFu, 0xFFFFFFFFu);
+      if (valid) vv = *reinterpret_cast<const uint4*>(valid + p0);
+      const uint8_t* vb = reinterpret_cast<const uint8_t*>(&vv);
+      uint4 out;
+      uint8_t* ob = reinterpret_cast<uint8_t*>(&out);
+#pragma unroll
+      for (int i = 0; i < 16; ++i) {
+        const int64_t p = p0 + i;
+        while (c + 1 < n_cont && p >= offs[c + 1]) ++c;
+        const int32_t b = cb[c];
+        const int64_t t = p - offs[c];
+        ob[i] = (b >= 0 && t >= b && vb[i] != 0) ? 1 : 0;
+      }
+      *reinterpret_cast<uint4*>(mask + p0) = out;
+    } else {
+      const int64_t last = p0 + 16 < hi ? p0 + 16 : hi;
+      for (int64_t p = first; p < last; ++p) {
+        while (c + 1 < n_cont && p >= offs[c + 1]) ++c;
+        mask[p] = mask_byte(cb, offs, c, p, valid);
+      }
+    }
+  }
+}
+
+}  // namespace
+}  // namespace hdl
+
+using namespace hdl;
+
+extern "C" hdl_status hdl_assign_continuations(const int32_t* n_selected,
+                                               const int32_t* branch_pos, int32_t n_roots,
+                                               int32_t k, const int32_t* conts_per_root,
+                                               int32_t extra_to_higher, int32_t* cont_branch,
+                                               int64_t n_cont_capacity, void* cuda_stream) {
+  if (n_roots < 0 || k < 0 || n_cont_capacity < 0) return HDL_ERR_INVALID_ARG;
+  if (k > 16) return HDL_ERR_UNSUPPORTED;
+  if (n_roots == 0 || n_cont_capacity == 0) return HDL_OK;
+  if (!n_selected || !conts_per_root || !cont_branch || (k > 0 && !branch_pos))
+    return HDL_ERR_INVALID_ARG;
+  if (!aligned_to(n_selected, 4) || !aligned_to(conts_per_root, 4) ||
+      !aligned_to(cont_branch, 4) || (branch_pos && !aligned_to(branch_pos, 4)))
+    return HDL_ERR_INVALID_ARG;
+  assign_continuations_kernel<<<1, kAssignThreads, 0, as_stream(cuda_stream)>>>(
+      n_selected, branch_pos, n_roots, k, conts_per_root, extra_to_higher, cont_branch,
+      n_cont_capacity);
+  return launch_status();
+}
+
+extern "C" hdl_status hdl_suffix_mask(const int32_t* cont_branch, const int64_t* cont_offsets,
+                                      int32_t n_cont, const uint8_t* cont_valid, uint8_t* mask,
+                                      int64_t mask_len, void* cuda_stream) {
+  if (n_cont < 0 || mask_len < 0) return HDL_ERR_INVALID_ARG;
+  if (n_cont == 0 || mask_len == 0) return HDL_OK;
+  if (!cont_branch || !cont_offsets || !mask) return HDL_ERR_INVALID_ARG;
+  if (!aligned_to(cont_branch, 4) || !aligned_to(cont_offsets, 8)) return HDL_ERR_INVALID_ARG;
+  const bool vec = aligned_to(mask, 16) && (cont_valid == nullptr || aligned_to(cont_valid, 16));
+  const int sms = current_sm_count();
+  if (sms <= 0) return HDL_ERR_CUDA;
+  const int64_t chunks = ceil_div(mask_len, 16);
+  const int64_t blocks = ceil_div(chunks, kMaskThreads);
+  const int grid = static_cast<int>(blocks < 4 * sms ? (blocks > 0 ? blocks : 1) : 4 * sms);
+  cudaStream_t st = as_stream(cuda_stream);
+  if (vec)
+    suffix_mask_kernel<true><<<grid, kMaskThreads, 0, st>>>(cont_branch, cont_offsets, n_cont,
+                                                            cont_valid, mask, mask_len);
+  else
+    suffix_mask_kernel<false><<<grid, kMaskThreads, 0, st>>>(cont_branch, cont_offsets, n_cont,
+                                                             cont_valid, mask, mask_len);
+  return launch_status();
+}

@@ -1,0 +1,507 @@
+// Hindsight re-scoring on the tcgen05 tensor cores (Section 3.1, Eq.
+// hindsight-contexts; Section 3.2, Eq. div).
+//
+// For every row h of the stacked hidden states [H_orig; H_hind] (2N x d) the
+// kernel needs log softmax(h W^T)[y] = z_y - log sum_v exp(z_v), z = h W^T.
+// The [2N, V] logits are never stored: a persistent, warp-specialised kernel
+// computes 128 x 256 logit tiles into TMEM and folds each tile straight into a
+// running (max, sum of exponentials) per row, picking the target logit out of
+// the tile that holds it.
+//
+// Work unit = (M-tile of 128 rows of one context, vocabulary chunk of
+// kTilesPerChunk 256-wide tiles).  Each unit writes one partial (max, sum)
+// per row; a second, tiny kernel merges the chunks, forms both log-probs and
+// |Delta|.  Splitting the vocabulary keeps the set of tiles that the ~150
+// concurrently running units touch small enough to stay in L2 (grouped
+// rasterisation: kGroupM M-tiles x a few chunks at a time), instead of every
+// CTA streaming its own 128 x d slice of H for the whole vocabulary.
+//
+// Roles inside a CTA of 192 threads:
+//   warp 0      TMA producer: H tile (128 x 128 B) + W tile (256 x 128 B) per
+//               K step into a kStages-deep shared-memory ring;
+//   warp 1      TMEM allocator and MMA issuer (one thread): 4 x
+//               tcgen05.mma 128x256x(32 B) per K step, accumulators in two
+//               256-column TMEM buffers so the epilogue of tile j overlaps
+//               the MMAs of tile j+1;
+//   warps 2..5  epilogue: one accumulator row per thread (TMEM lane), 32
+//               columns per tcgen05.ld, online log-sum-exp in base 2 and the
+//               target-column select.
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <cudaTypedefs.h>
+
+#include <cmath>
+#include <cstdint>
+#include <mutex>
+
+#include "hdl.h"
+#include "hdl_internal.h"
+#include "ptx_sm103.cuh"
+
+namespace hdl {
+namespace {
+
+constexpr int kBM = 128;             // rows per tile = TMEM lanes
+constexpr int kBN = 256;             // vocabulary columns per tile
+constexpr int kRowBytes = 128;       // K bytes per stage (one 128-byte swizzle row)
+constexpr int kStages = 4;
+constexpr int kTilesPerChunk = 16;   // 4096 vocabulary entries per unit
+constexpr int kGroupM = 16;          // M-tiles per rasterisation group
+constexpr int kThreads = 192;
+constexpr int kAStage = kBM * kRowBytes;        // 16 KiB
+constexpr int kBStage = kBN * kRowBytes;        // 32 KiB
+constexpr int kStageBytes = kAStage + kBStage;  // 48 KiB
+constexpr int kMmaPerStage = kRowBytes / 32;    // 32 bytes of K per MMA
+constexpr int kTmemCols = 2 * kBN;              // two accumulator buffers
+constexpr int kBarOffset = kStages * kStageBytes;
+constexpr int kSmemBytes = kBarOffset + 256 + 1024;   // + barriers + alignment slack
+constexpr uint64_t kDefaultTimeoutNs = 4000000000ull;   // 4 s per wait
+constexpr float kLog2e = 1.4426950408889634f;
+constexpr float kLn2 = 0.6931471805599453f;
+
+struct RescoreArgs {
+  const int32_t* targets;
+  float2* part;        // [num_chunks][2N] partial (max in log2 units, sum)
+  float* zt;           // [2N] target logit
+  uint32_t* status;
+  int64_t n_tokens;    // N rows per context
+  int32_t vocab;
+  int32_t num_kb;      // K steps (d * esize / 128)
+  int32_t num_m_ctx;   // M-tiles per context
+  int32_t num_m;       // M-tiles, both contexts
+  int32_t num_vt;      // vocabulary tiles
+  int32_t num_chunks;
+  int32_t num_units;
+  uint64_t timeout_ns;
+};
+
+struct Unit {
+  int ctx;       // 0 = original context, 1 = hindsight context
+  int row0;      // first row of the tile within its context
+  int chunk;
+  int vt0, vt1;  // vocabulary tiles [vt0, vt1)
+};
+
+// Grouped rasterisation: consecutive units run through kGroupM M-tiles
+// first, then the chunks, so concurrently running units share both their
+// H tiles and their W tiles in L2.
+__device__ __forceinline__ Unit decode_unit(int u, const RescoreArgs& a) {
+  const int per_group = kGroupM * a.num_chunks;
+  const int g = u / per_group;
+  const int first = g * kGroupM;
+  const int gsz = min(a.num_m - first, kGroupM);
+  const int r = u - g * per_group;
+  const int mt = first + r % gsz;
+  Unit w;
+  w.chunk = r / gsz;
+  w.ctx = mt >= a.num_m_ctx ? 1 : 0;
+  w.row0 = (mt - w.ctx * a.num_m_ctx) * kBM;
+  w.vt0 = w.chunk * kTilesPerChunk;
+  w.vt1 = min(w.vt0 + kTilesPerChunk, a.num_vt);
+  return w;
+}
+
+// Fold 32 logits into the running base-2 (max, sum) of one row.
+__device__ __forceinline__ void lse_fold(const float (&x)[32], float& m2, float& s) {
+  float c[16];
+#pragma unroll
+  for (int j = 0; j < 16; ++j) c[j] = fmaxf(x[j], x[j + 16]);
+#pragma unroll
+  for (int w = 8; w >= 1; w >>= 1)
+#pragma unroll
+    for (int j = 0; j < w; ++j) c[j] = fmaxf(c[j], c[j + w]);
+  const float m_new = fmaxf(m2, c[0] * kLog2e);
+  float acc[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+  for (int j = 0; j < 32; ++j) acc[j & 3] += ex2_approx(fmaf(x[j], kLog2e, -m_new));
+  s = fmaf(s, ex2_approx(m2 - m_new), (acc[0] + acc[1]) + (acc[2] + acc[3]));
+  m2 = m_new;
+}
+
+template <bool kTf32>
+__global__ void __launch_bounds__(kThreads, 1)
+    rescore_lse_kernel(const __grid_constant__ CUtensorMap tm_h0,
+                       const __grid_constant__ CUtensorMap tm_h1,
+                       const __grid_constant__ CUtensorMap tm_w, const RescoreArgs a) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>(
+      (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
+  const uint32_t sbase = smem_addr(smem);
+  const uint32_t sA = sbase;                       // kStages x 16 KiB
+  const uint32_t sB = sbase + kStages * kAStage;   // kStages x 32 KiB
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + kBarOffset);
+  const uint32_t bar0 = smem_addr(bars);
+  auto full_bar = [&](int s) { return bar0 + 8u * s; };
+  auto empty_bar = [&](int s) { return bar0 + 8u * (kStages + s); };
+  auto tfull_bar = [&](int b) { return bar0 + 8u * (2 * kStages + b); };
+  auto tempty_bar = [&](int b) { return bar0 + 8u * (2 * kStages + 2 + b); };
+  const uint32_t done_bar = bar0 + 8u * (2 * kStages + 4);
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + kBarOffset + 8 * (2 * kStages + 5));
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kStages; ++s) {
+      mbar_init(full_bar(s), 1);
+      mbar_init(empty_bar(s), 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(tfull_bar(b), 1);
+      mbar_init(tempty_bar(b), 4);
+    }
+    mbar_init(done_bar, 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+  }
+  if (warp == 0 && lane == 0) {
+    tma_prefetch_desc(&tm_h0);
+    tma_prefetch_desc(&tm_h1);
+    tma_prefetch_desc(&tm_w);
+  }
+  if (warp == 1) tmem_alloc(smem_addr(tmem_slot), kTmemCols);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+
+  PipeCtl ctl{abort_flag, a.status, a.timeout_ns};
+
+  if (warp == 0) {
+    // ------------------------------------------------------ TMA producer
+    if (lane == 0) {
+      int stage = 0;
+      uint32_t phase = 0, pend = 0, pend_par = 0;
+      bool ok = true;
+      for (int u = blockIdx.x; ok && u < a.num_units; u += gridDim.x) {
+        const Unit w = decode_unit(u, a);
+        const CUtensorMap* tmA = w.ctx ? &tm_h1 : &tm_h0;
+        for (int vt = w.vt0; ok && vt < w.vt1; ++vt) {
+          for (int kb = 0; kb < a.num_kb; ++kb) {
+            if (!mbar_wait_bounded(empty_bar(stage), phase ^ 1u, ctl, kRoleProducer)) {
+              ok = false;
+              break;
+            }
+            mbar_arrive_expect_tx(full_bar(stage), kStageBytes);
+            const int32_t kx = kb * (kRowBytes / (kTf32 ? 4 : 2));
+            tma_load_2d(sA + stage * kAStage, tmA, kx, w.row0, full_bar(stage));
+            tma_load_2d(sB + stage * kBStage, &tm_w, kx, vt * kBN, full_bar(stage));
+            pend |= 1u << stage;
+            pend_par = (pend_par & ~(1u << stage)) | (phase << stage);
+            if (++stage == kStages) {
+              stage = 0;
+              phase ^= 1u;
+            }
+          }
+        }
+      }
+      if (!ok) {
+        // Aborted: let the copies already issued land before the CTA exits.
+        for (int s = 0; s < kStages; ++s)
+          if ((pend >> s) & 1u) mbar_wait_drain(full_bar(s), (pend_par >> s) & 1u, 100000000ull);
+      }
+    }
+    __syncwarp();
+  } else if (warp == 1) {
+    // --------------------------------------------------------- MMA issuer
+    if (lane == 0) {
+      constexpr uint32_t idesc = make_idesc(kTf32 ? 2u : 1u, kBM, kBN);
+      int stage = 0;
+      uint32_t phase = 0, tile = 0;
+      bool ok = true;
+      for (int u = blockIdx.x; ok && u < a.num_units; u += gridDim.x) {
+        const Unit w = decode_unit(u, a);
+        for (int vt = w.vt0; ok && vt < w.vt1; ++vt, ++tile) {
+          const uint32_t buf = tile & 1u, use = (tile >> 1) & 1u;
+          if (!mbar_wait_bounded(tempty_bar(buf), use ^ 1u, ctl, kRoleMma)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t d_tmem = tmem_base + buf * kBN;
+          for (int kb = 0; kb < a.num_kb; ++kb) {
+            if (!mbar_wait_bounded(full_bar(stage), phase, ctl, kRoleMma)) {
+              ok = false;
+              break;
+            }
+            tc_fence_after();
+            const uint32_t a_addr = sA + stage * kAStage;
+            const uint32_t b_addr = sB + stage * kBStage;
+#pragma unroll
+            for (int kk = 0; kk < kMmaPerStage; ++kk)
+              tc_mma<kTf32>(d_tmem, smem_desc_sw128(a_addr + 32 * kk),
+                            smem_desc_sw128(b_addr + 32 * kk), idesc,
+                            (kb | kk) != 0 ? 1u : 0u);
+            tc_commit(empty_bar(stage));
+            if (++stage == kStages) {
+              stage = 0;
+              phase ^= 1u;
+            }
+          }
+          if (ok) tc_commit(tfull_bar(buf));
+        }
+      }
+      // Every MMA issued above must finish before TMEM is released.
+      tc_commit(done_bar);
+      mbar_wait_drain(done_bar, 0, 1000000000ull);
+    }
+    __syncwarp();
+  } else {
+    // ----------------------------------------------------------- epilogue
+    const int q = warp & 3;              // TMEM lane quadrant of this warp
+    const int r_in_tile = q * 32 + lane;
+    const uint32_t lane_addr = static_cast<uint32_t>(q * 32) << 16;
+    uint32_t tile = 0;
+    bool ok = true;
+    for (int u = blockIdx.x; ok && u < a.num_units; u += gridDim.x) {
+      const Unit w = decode_unit(u, a);
+      const int64_t row = static_cast<int64_t>(w.row0) + r_in_tile;
+      const bool in_range = row < a.n_tokens;
+      const int32_t y = in_range ? __ldg(a.targets + row) : -1;
+      float m2 = -INFINITY, s = 0.f, zt = 0.f;
+      bool found = false;
+      for (int vt = w.vt0; vt < w.vt1; ++vt, ++tile) {
+        const uint32_t buf = tile & 1u, use = (tile >> 1) & 1u;
+        bool got = mbar_wait_bounded(tfull_bar(buf), use, ctl, kRoleEpilogue);
+        if (!__all_sync(0xffffffffu, got)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const int v0 = vt * kBN;
+        const int ncols = min(kBN, a.vocab - v0);
+        const uint32_t taddr = tmem_base + lane_addr + buf * kBN;
+#pragma unroll
+        for (int cc = 0; cc < kBN / 32; ++cc) {
+          if (cc * 32 < ncols) {
+            float x[32];
+            __syncwarp();  // tcgen05.ld is warp-collective: reconverge first
+            tmem_load32(taddr + cc * 32, x);
+            if (cc * 32 + 32 > ncols) {
+#pragma unroll
+              for (int j = 0; j < 32; ++j)
+                if (cc * 32 + j >= ncols) x[j] = -INFINITY;
+            }
+            lse_fold(x, m2, s);
+            const int rel = y - (v0 + cc * 32);
+            if (static_cast<unsigned>(rel) < 32u) {
+#pragma unroll
+              for (int j = 0; j < 32; ++j)
+                if (j == rel) zt = x[j];
+              found = true;
+            }
+          }
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(tempty_bar(buf));
+      }
+      if (ok && in_range) {
+        const int64_t rows_total = 2 * a.n_tokens;
+        const int64_t g = w.ctx * a.n_tokens + row;
+        a.part[static_cast<int64_t>(w.chunk) * rows_total + g] = make_float2(m2, s);
+        if (found) a.zt[g] = zt;
+      }
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem_base, kTmemCols);
+  }
+}
+
+// Merge the per-chunk partials of both contexts of token t and write
+// log p^0, log p^H and |Delta| (Eq. div).
+__global__ void __launch_bounds__(256)
+    rescore_merge_kernel(const float2* __restrict__ part, const float* __restrict__ zt,
+                         const int32_t* __restrict__ targets, int64_t n, int32_t vocab,
+                         int32_t num_chunks, float* __restrict__ lp0,
+                         float* __restrict__ lp1, float* __restrict__ delta,
+                         uint32_t* status) {
+  const int64_t rows_total = 2 * n;
+  for (int64_t t = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; t < n;
+       t += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+    float lp[2];
+#pragma unroll
+    for (int ctx = 0; ctx < 2; ++ctx) {
+      const int64_t g = ctx * n + t;
+      float M = -INFINITY;
+      for (int c = 0; c < num_chunks; ++c) M = fmaxf(M, part[c * rows_total + g].x);
+      float S = 0.f;
+      for (int c = 0; c < num_chunks; ++c) {
+        const float2 p = part[c * rows_total + g];
+        S += p.y * exp2f(p.x - M);
+      }
+      lp[ctx] = zt[g] - (M + log2f(S)) * kLn2;
+    }
+    const int32_t y = targets[t];
+    if (y < 0 || y >= vocab) {
+      lp[0] = lp[1] = __int_as_float(0x7fc00000);
+      atomicOr(status, kStatusBadTarget);
+    }
+    lp0[t] = lp[0];
+    lp1[t] = lp[1];
+    if (delta) delta[t] = fabsf(lp[1] - lp[0]);
+  }
+}
+
+struct Geometry {
+  int64_t n;
+  int esize;
+  int num_kb, num_m_ctx, num_m, num_vt, num_chunks;
+  int64_t num_units;
+  size_t zt_off, part_off, total;
+};
+
+Geometry geometry(int64_t n, int32_t d, int32_t vocab, hdl_dtype dt) {
+  Geometry g{};
+  g.n = n;
+  g.esize = dt == HDL_F32 ? 4 : 2;
+  g.num_kb = static_cast<int>(static_cast<int64_t>(d) * g.esize / kRowBytes);
+  g.num_m_ctx = static_cast<int>(ceil_div(n, kBM));
+  g.num_m = 2 * g.num_m_ctx;
+  g.num_vt = static_cast<int>(ceil_div(vocab, kBN));
+  g.num_chunks = static_cast<int>(ceil_div(g.num_vt, kTilesPerChunk));
+  g.num_units = static_cast<int64_t>(g.num_m) * g.num_chunks;
+  g.zt_off = 256;
+  g.part_off = g.zt_off + align_up(static_cast<size_t>(2 * n) * sizeof(float), 256);
+  g.total = g.part_off + static_cast<size_t>(g.num_chunks) * static_cast<size_t>(2 * n) * sizeof(float2);
+  return g;
+}
+
+PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000,
+                                         cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  });
+  return fn;
+}
+
+// 2-D row-major [rows, d] operand, boxes of (128 bytes of K) x box_rows,
+// 128-byte swizzle; rows past the end read as zeros.
+bool make_operand_map(CUtensorMap* m, const void* ptr, int64_t rows, int32_t d, int esize,
+                      int box_rows) {
+  auto enc = tensor_map_encoder();
+  if (!enc) return false;
+  cuuint64_t dims[2] = {static_cast<cuuint64_t>(d), static_cast<cuuint64_t>(rows)};
+  cuuint64_t strides[1] = {static_cast<cuuint64_t>(d) * esize};
+  cuuint32_t box[2] = {static_cast<cuuint32_t>(kRowBytes / esize),
+                       static_cast<cuuint32_t>(box_rows)};
+  cuuint32_t estr[2] = {1, 1};
+  const CUresult r = enc(m, esize == 2 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT32,
+                         2, const_cast<void*>(ptr), dims, strides, box, estr,
+                         CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                         CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS;
+}
+
+hdl_status check_shape(int64_t n_tokens, int32_t d, int32_t vocab, hdl_dtype dt) {
+  if (n_tokens < 0 || d <= 0 || vocab <= 0) return HDL_ERR_INVALID_ARG;
+  if (dt != HDL_BF16 && dt != HDL_F32) return HDL_ERR_INVALID_ARG;
+  if (d % 64 != 0 || d > 65536) return HDL_ERR_UNSUPPORTED;
+  if (n_tokens > (int64_t{1} << 30) || vocab > (1 << 30)) return HDL_ERR_UNSUPPORTED;
+  const Geometry g = geometry(n_tokens, d, vocab, dt);
+  if (g.num_units >= (int64_t{1} << 31)) return HDL_ERR_UNSUPPORTED;
+  return HDL_OK;
+}
+
+}  // namespace
+}  // namespace hdl
+
+using namespace hdl;
+
+extern "C" size_t hdl_rescore_workspace_bytes(int64_t n_tokens, int32_t d, int32_t vocab,
+                                              hdl_dtype dt) {
+  if (check_shape(n_tokens, d, vocab, dt) != HDL_OK) return 0;
+  return geometry(n_tokens, d, vocab, dt).total;
+}
+
+extern "C" hdl_status hdl_rescore(const void* h_orig, const void* h_hind, const void* w_lmhead,
+                                  hdl_dtype dt, const int32_t* targets, int64_t n_tokens,
+                                  int32_t d, int32_t vocab, float* logp_orig, float* logp_hind,
+                                  float* delta, void* workspace, size_t workspace_bytes,
+                                  void* cuda_stream) {
+  const hdl_status sh = check_shape(n_tokens, d, vocab, dt);
+  if (sh != HDL_OK) return sh;
+  if (n_tokens == 0) return HDL_OK;
+  if (!h_orig || !h_hind || !w_lmhead || !targets || !logp_orig || !logp_hind)
+    return HDL_ERR_INVALID_ARG;
+  if (!aligned_to(h_orig, 16) || !aligned_to(h_hind, 16) || !aligned_to(w_lmhead, 16) ||
+      !aligned_to(targets, 4) || !aligned_to(logp_orig, 4) || !aligned_to(logp_hind, 4) ||
+      (delta && !aligned_to(delta, 4)))
+    return HDL_ERR_INVALID_ARG;
+  const Geometry g = geometry(n_tokens, d, vocab, dt);
+  if (!workspace || !aligned_to(workspace, 256) || workspace_bytes < g.total)
+    return HDL_ERR_WORKSPACE;
+
+  CUtensorMap tm_h0, tm_h1, tm_w;
+  if (!make_operand_map(&tm_h0, h_orig, n_tokens, d, g.esize, kBM) ||
+      !make_operand_map(&tm_h1, h_hind, n_tokens, d, g.esize, kBM) ||
+      !make_operand_map(&tm_w, w_lmhead, vocab, d, g.esize, kBN))
+    return HDL_ERR_CUDA;
+
+  uint8_t* ws = static_cast<uint8_t*>(workspace);
+  RescoreArgs a{};
+  a.targets = targets;
+  a.status = reinterpret_cast<uint32_t*>(ws);
+  a.zt = reinterpret_cast<float*>(ws + g.zt_off);
+  a.part = reinterpret_cast<float2*>(ws + g.part_off);
+  a.n_tokens = n_tokens;
+  a.vocab = vocab;
+  a.num_kb = g.num_kb;
+  a.num_m_ctx = g.num_m_ctx;
+  a.num_m = g.num_m;
+  a.num_vt = g.num_vt;
+  a.num_chunks = g.num_chunks;
+  a.num_units = static_cast<int32_t>(g.num_units);
+  a.timeout_ns = kDefaultTimeoutNs;
+
+  cudaStream_t st = as_stream(cuda_stream);
+  if (cudaMemsetAsync(a.status, 0, sizeof(uint32_t), st) != cudaSuccess) return HDL_ERR_CUDA;
+
+  const int sms = current_sm_count();
+  if (sms <= 0) return HDL_ERR_CUDA;
+  const int grid = static_cast<int>(g.num_units < sms ? g.num_units : sms);
+  if (dt == HDL_F32) {
+    if (cudaFuncSetAttribute(rescore_lse_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             kSmemBytes) != cudaSuccess)
+      return HDL_ERR_CUDA;
+    rescore_lse_kernel<true><<<grid, kThreads, kSmemBytes, st>>>(tm_h0, tm_h1, tm_w, a);
+  } else {
+    if (cudaFuncSetAttribute(rescore_lse_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             kSmemBytes) != cudaSuccess)
+      return HDL_ERR_CUDA;
+    rescore_lse_kernel<false><<<grid, kThreads, kSmemBytes, st>>>(tm_h0, tm_h1, tm_w, a);
+  }
+  if (launch_status() != HDL_OK) return HDL_ERR_CUDA;
+
+  const int64_t mblocks = ceil_div(n_tokens, 256);
+  const int mgrid = static_cast<int>(mblocks < 8 * sms ? mblocks : 8 * sms);
+  rescore_merge_kernel<<<mgrid, 256, 0, st>>>(a.part, a.zt, targets, n_tokens, vocab,
+                                              g.num_chunks, logp_orig, logp_hind, delta,
+                                              a.status);
+  return launch_status();
+}
+
+extern "C" hdl_status hdl_device_status(const void* workspace, size_t workspace_bytes,
+                                        void* cuda_stream, uint32_t* raw_word) {
+  if (!workspace || workspace_bytes < sizeof(uint32_t)) return HDL_ERR_INVALID_ARG;
+  if (cudaStreamSynchronize(as_stream(cuda_stream)) != cudaSuccess) return HDL_ERR_CUDA;
+  uint32_t word = 0;
+  if (cudaMemcpy(&word, workspace, sizeof(word), cudaMemcpyDeviceToHost) != cudaSuccess)
+    return HDL_ERR_CUDA;
+  if (raw_word) *raw_word = word;
+  if (word & kStatusTimeout) return HDL_ERR_TIMEOUT;
+  if (word & kStatusBadTarget) return HDL_ERR_BAD_TARGET;
+  return HDL_OK;
+}

@@ -1,0 +1,68 @@
+"""Bridges between the generated workloads, the CPU oracle and the tolerances
+of the parity tests (test code: the library never imports this)."""
+from __future__ import annotations
+
+import numpy as np
+import torch
+
+import oracle
+
+# Log-probability tolerance: |err| <= ATOL + RTOL * |ref|.
+LP_ATOL = 1e-3
+LP_RTOL = 1e-3
+# End-to-end selection may differ only at positions whose reference score is
+# within this band of the root's k-th selected score.
+SELECT_BAND = 2e-3
+
+
+def to_f64(t: torch.Tensor) -> np.ndarray:
+    """Exact float64 copy of a bf16 or fp32 tensor (via the oracle's widening)."""
+    t = t.detach().cpu().contiguous()
+    if t.dtype == torch.bfloat16:
+        return oracle.widen(t.view(torch.int16).numpy(), "bf16")
+    if t.dtype == torch.float32:
+        return oracle.widen(t.numpy(), "f32")
+    raise TypeError(t.dtype)
+
+
+def oracle_logprobs(h64: np.ndarray, w64: np.ndarray, y: np.ndarray, block: int = 1024):
+    """oracle.target_logprobs over row blocks (each row is independent)."""
+    out = np.empty(h64.shape[0])
+    for s in range(0, h64.shape[0], block):
+        out[s:s + block] = oracle.target_logprobs(h64[s:s + block], w64, y[s:s + block])
+    return out
+
+
+def assert_logp_close(got, ref, what=""):
+    got = np.asarray(got, np.float64)
+    ref = np.asarray(ref, np.float64)
+    err = np.abs(got - ref)
+    bound = LP_ATOL + LP_RTOL * np.abs(ref)
+    bad = ~(err <= bound)
+    assert not bad.any(), (f"{what}: {bad.sum()} of {bad.size} outside tolerance; "
+                           f"max err {err.max():.3e} at {int(err.argmax())}")
+    return float(err.max()) if err.size else 0.0
+
+
+def sample_rows(n: int, count: int, seed: int = 0) -> np.ndarray:
+    """First, last and random rows (sorted, unique)."""
+    rng = np.random.default_rng(seed)
+    pick = set([0, n - 1]) | set(rng.integers(0, n, size=count).tolist())
+    return np.array(sorted(pick), dtype=np.int64)
+
+
+def check_selection_band(gpu_pos, gpu_nsel, ref_delta, valid, offs, k, band=SELECT_BAND):
+    """GPU branch sets vs. the oracle's on the oracle's scores: equal except at
+    positions whose reference score lies within ``band`` of the k-th value."""
+    pos, nsel, _ = oracle.select_branches(ref_delta, valid, offs, k)
+    gpu_pos = np.asarray(gpu_pos)
+    for r in range(len(offs) - 1):
+        assert int(gpu_nsel[r]) == int(nsel[r]), (r, gpu_nsel[r], nsel[r])
+        n = int(nsel[r])
+        if n == 0:
+            continue
+        a = set(gpu_pos[r, :n].tolist())
+        b = set(pos[r, :n].tolist())
+        kth = ref_delta[offs[r] + pos[r, n - 1]]
+        for t in a ^ b:
+            assert abs(ref_delta[offs[r] + t] - kth) <= band, (r, t, ref_delta[offs[r] + t], kth)

@@ -1,0 +1,113 @@
+"""Re-scoring parity (Section 3.1-3.2): the tcgen05 kernel against the fp64
+oracle, element by element, on shapes that cover every tile edge."""
+import numpy as np
+import pytest
+import torch
+
+import hdl_synth
+from tests.helpers import assert_logp_close, oracle_logprobs, to_f64
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def hdl():
+    import __graft_entry__
+    __graft_entry__.build()
+    import paper_2609_36864_gb300 as m
+    return m
+
+
+def run_and_check(hdl, wl, what):
+    lp0, lp1, delta, ws = hdl.hdl_rescore(wl.h_orig, wl.h_hind, wl.w, wl.targets)
+    code, raw = hdl.hdl_device_status(ws)
+    assert code == hdl.HDL_OK, (code, hex(raw))
+    W = to_f64(wl.w)
+    y = wl.targets.cpu().numpy()
+    r0 = oracle_logprobs(to_f64(wl.h_orig), W, y)
+    r1 = oracle_logprobs(to_f64(wl.h_hind), W, y)
+    e0 = assert_logp_close(lp0.cpu().numpy(), r0, what + " orig")
+    e1 = assert_logp_close(lp1.cpu().numpy(), r1, what + " hind")
+    d = delta.cpu().numpy().astype(np.float64)
+    assert np.array_equal(d, np.abs(lp1.cpu().numpy() - lp0.cpu().numpy()).astype(np.float64))
+    return max(e0, e1), r0, r1, d
+
+
+# (tokens, d, V, dtype): rows around the 128-row tile, vocabularies around the
+# 256-column tile and the 4096-column chunk, several K steps.
+SHAPES = [
+    (1, 64, 1, "bf16"),        # one row, one word: log p = 0
+    (5, 64, 300, "bf16"),      # one partial vocabulary tile
+    (127, 128, 256, "bf16"),
+    (128, 128, 512, "bf16"),
+    (129, 192, 257, "bf16"),   # ragged rows and a 1-column last tile
+    (300, 256, 4097, "bf16"),  # second chunk holds a single column
+    (700, 512, 9000, "bf16"),
+    (1000, 1024, 8192, "bf16"),
+    (200, 256, 5000, "f32"),   # tf32 path
+    (513, 64, 4096, "f32"),
+]
+
+
+@pytest.mark.parametrize("n,d,V,dt", SHAPES)
+def test_rescore_shapes(hdl, n, d, V, dt):
+    spec = hdl_synth.small_spec(f"s{n}_{d}_{V}", n_roots=1, t_lo=n, t_hi=n, d=d, vocab=V,
+                                dtype=dt, seed=n + V)
+    wl = hdl_synth.generate(spec, device="cuda")
+    err, r0, _, _ = run_and_check(hdl, wl, str((n, d, V, dt)))
+    if V == 1:
+        assert np.all(r0 == 0.0)
+
+
+def test_rescore_identical_contexts_bitwise(hdl):
+    """Delta = 0 exactly when both contexts carry the same hidden states, and
+    the two log-prob rows are bit-identical (same arithmetic for both)."""
+    spec = hdl_synth.small_spec("same", n_roots=2, t_lo=300, t_hi=400, d=256, vocab=6000)
+    wl = hdl_synth.generate(spec, device="cuda")
+    lp0, lp1, delta, ws = hdl.hdl_rescore(wl.h_orig, wl.h_orig.clone(), wl.w, wl.targets)
+    assert hdl.hdl_device_status(ws)[0] == hdl.HDL_OK
+    assert torch.equal(lp0, lp1)
+    assert torch.all(delta == 0)
+
+
+def test_rescore_invariants(hdl):
+    """log p <= 0 and the normaliser is shared: summing p over every target
+    of one row gives 1."""
+    V, d = 3000, 128
+    g = torch.Generator(device="cuda").manual_seed(3)
+    w = (torch.randn(V, d, generator=g, device="cuda") * 0.05).to(torch.bfloat16)
+    h = torch.randn(1, d, generator=g, device="cuda").to(torch.bfloat16).repeat(V, 1)
+    y = torch.arange(V, dtype=torch.int32, device="cuda")
+    lp0, lp1, _, _ = hdl.hdl_rescore(h, h, w, y)
+    lp = lp0.double()
+    assert torch.all(lp <= 1e-6)
+    assert abs(torch.exp(lp).sum().item() - 1.0) < 1e-4
+
+
+def test_rescore_bad_target_reported(hdl):
+    spec = hdl_synth.small_spec("bad", n_roots=1, t_lo=50, t_hi=50, d=64, vocab=500)
+    wl = hdl_synth.generate(spec, device="cuda")
+    y = wl.targets.clone()
+    y[7] = 500
+    y[9] = -1
+    lp0, lp1, delta, ws = hdl.hdl_rescore(wl.h_orig, wl.h_hind, wl.w, y)
+    code, raw = hdl.hdl_device_status(ws)
+    assert code == hdl.HDL_ERR_BAD_TARGET and (raw & 2)
+    bad = torch.isnan(lp0).cpu()
+    assert bad[7] and bad[9] and bad.sum() == 2
+    # the next call on the same workspace starts from a clear status word
+    lp0, lp1, delta, ws = hdl.hdl_rescore(wl.h_orig, wl.h_hind, wl.w, wl.targets, workspace=ws)
+    assert hdl.hdl_device_status(ws)[0] == hdl.HDL_OK
+
+
+def test_rescore_outputs_independent_of_stream_and_repeat(hdl):
+    spec = hdl_synth.small_spec("rep", n_roots=3, t_lo=100, t_hi=400, d=256, vocab=5000)
+    wl = hdl_synth.generate(spec, device="cuda")
+    a = hdl.hdl_rescore(wl.h_orig, wl.h_hind, wl.w, wl.targets)
+    s = torch.cuda.Stream()
+    s.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(s):
+        b = hdl.hdl_rescore(wl.h_orig, wl.h_hind, wl.w, wl.targets, stream=s)
+    s.synchronize()
+    for x, y in zip(a[:3], b[:3]):
+        assert torch.equal(x, y)

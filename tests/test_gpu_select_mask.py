@@ -1,0 +1,184 @@
+"""Selection, allocation and mask kernels: bit-exact against the oracle when
+fed the same scores, offsets and masks (Sections 3.2, 3.3, 4.1, 4.4)."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def hdl():
+    import __graft_entry__
+    __graft_entry__.build()
+    import paper_2609_36864_gb300 as m
+    return m
+
+
+def make_roots(lengths, seed, tie_levels=None, nan_frac=0.0, invalid_frac=0.2):
+    rng = np.random.default_rng(seed)
+    offs = np.concatenate([[0], np.cumsum(lengths)]).astype(np.int64)
+    N = int(offs[-1])
+    if tie_levels:
+        delta = (rng.integers(0, tie_levels, size=N) * 0.25).astype(np.float32)
+    else:
+        delta = rng.exponential(size=N).astype(np.float32)
+    if nan_frac:
+        delta[rng.random(N) < nan_frac] = np.nan
+    valid = (rng.random(N) >= invalid_frac).astype(np.uint8)
+    return delta, valid, offs
+
+
+def gpu_select(hdl, delta, valid, offs, k, **kw):
+    d = torch.from_numpy(delta).cuda()
+    v = None if valid is None else torch.from_numpy(valid).cuda()
+    o = torch.from_numpy(offs).cuda()
+    bp, ns, bd = hdl.hdl_select_branches(d, v, o, k, **kw)
+    return bp.cpu().numpy(), ns.cpu().numpy(), bd.cpu().numpy()
+
+
+def assert_select_equal(hdl, delta, valid, offs, k, **kw):
+    bp, ns, bd = gpu_select(hdl, delta, valid, offs, k, **kw)
+    pos, nsel, val = oracle.select_branches(delta.astype(np.float64), valid, offs, k, **kw)
+    assert np.array_equal(ns, nsel)
+    assert np.array_equal(bp, pos)
+    assert np.array_equal(bd.astype(np.float64), val, equal_nan=True)
+
+
+CASES = [
+    ([0, 1, 2, 3, 17, 100, 511, 513, 4096], 4, {}),
+    ([16384, 16384, 12000], 16, {}),                       # maximum k, long roots
+    ([3, 5, 1, 0, 2], 8, {}),                              # k > T
+    ([1000] * 40, 8, {}),                                  # many roots
+]
+
+
+@pytest.mark.parametrize("lengths,k,kw", CASES)
+def test_select_plain(hdl, lengths, k, kw):
+    for seed, ties in ((0, None), (1, 3), (2, 1)):        # distinct, heavy ties, all equal
+        delta, valid, offs = make_roots(lengths, seed, tie_levels=ties)
+        assert_select_equal(hdl, delta, valid, offs, k, **kw)
+        assert_select_equal(hdl, delta, None, offs, k, **kw)
+
+
+def test_select_nan_negative_zero_and_all_invalid(hdl):
+    delta, valid, offs = make_roots([200, 50, 300], 5, nan_frac=0.3)
+    delta[:10] = -0.0
+    delta[10:20] = 0.0
+    delta[20:25] = -1.5
+    delta[25] = np.inf
+    valid[offs[1]:offs[2]] = 0                            # a root with no candidate
+    for k in (0, 1, 5, 16):
+        assert_select_equal(hdl, delta, valid, offs, k)
+
+
+def test_select_window(hdl):
+    delta, valid, offs = make_roots([500, 20, 1000], 6)
+    for lo, hi in ((0, 0), (10, 0), (0, 100), (50, 60), (600, 0), (5, 3)):
+        assert_select_equal(hdl, delta, valid, offs, 8, lo=lo, hi=hi)
+
+
+@pytest.mark.parametrize("gap_mode", [0, 1])
+@pytest.mark.parametrize("min_gap", [1, 2, 7, 64])
+def test_select_spacing(hdl, gap_mode, min_gap):
+    for seed, ties in ((7, None), (8, 3)):
+        delta, valid, offs = make_roots([0, 5, 40, 300, 2048, 9000], seed, tie_levels=ties)
+        # cluster the large scores so that the spacing rule bites
+        delta[offs[4] + 100:offs[4] + 140] += 5
+        assert_select_equal(hdl, delta, valid, offs, 8, min_gap=min_gap, gap_mode=gap_mode)
+        assert_select_equal(hdl, delta, valid, offs, 16, min_gap=min_gap, gap_mode=gap_mode)
+
+
+def test_select_nonmonotone_offsets_are_empty(hdl):
+    delta, valid, offs = make_roots([100, 100], 9)
+    offs = np.array([0, 100, 50], dtype=np.int64)         # second root ends before it starts
+    bp, ns, bd = gpu_select(hdl, delta, valid, offs, 4)
+    assert ns[1] == 0 and np.all(bp[1] == -1)
+
+
+@pytest.mark.parametrize("extra_to_higher", [True, False])
+def test_assign_continuations(hdl, extra_to_higher):
+    rng = np.random.default_rng(11)
+    R, k = 300, 8
+    nsel = rng.integers(0, k + 1, size=R).astype(np.int32)
+    pos = np.full((R, k), -1, np.int32)
+    for r in range(R):
+        pos[r, :nsel[r]] = rng.choice(5000, size=nsel[r], replace=False)
+    conts = rng.integers(0, 20, size=R).astype(np.int32)
+    conts[:3] = [7, 7, 3]
+    ref = oracle.assign_continuations(nsel, pos, conts, extra_to_higher)
+    cb = hdl.hdl_assign_continuations(torch.from_numpy(nsel).cuda(), torch.from_numpy(pos).cuda(),
+                                      torch.from_numpy(conts).cuda(), extra_to_higher,
+                                      n_cont=int(conts.sum()))
+    assert np.array_equal(cb.cpu().numpy(), ref)
+
+
+def test_assign_paper_configs(hdl):
+    """2x2 -> 3+4, 2x1 -> 7, 4x2 -> 1+2 per root (Section 4.1, Table fork-ablation)."""
+    for roots, pts, C, counts in ((2, 2, 7, [4, 3]), (2, 1, 7, [7]), (4, 2, 3, [2, 1])):
+        nsel = torch.full((roots,), pts, dtype=torch.int32, device="cuda")
+        pos = torch.arange(roots * pts, dtype=torch.int32, device="cuda").view(roots, pts) * 10
+        conts = torch.full((roots,), C, dtype=torch.int32, device="cuda")
+        cb = hdl.hdl_assign_continuations(nsel, pos, conts, n_cont=roots * C).cpu().numpy()
+        for r in range(roots):
+            seg = cb[r * C:(r + 1) * C]
+            got = [int((seg == p).sum()) for p in pos[r].cpu().numpy()]
+            assert got == counts
+
+
+def test_assign_capacity_is_respected(hdl):
+    nsel = torch.tensor([2, 2], dtype=torch.int32, device="cuda")
+    pos = torch.tensor([[1, 2], [3, 4]], dtype=torch.int32, device="cuda")
+    conts = torch.tensor([7, 7], dtype=torch.int32, device="cuda")
+    out = torch.full((20,), -7, dtype=torch.int32, device="cuda")
+    hdl.hdl_assign_continuations(nsel, pos, conts, cont_branch=out[:10])
+    o = out.cpu().numpy()
+    assert np.array_equal(o[:10], [1, 1, 1, 1, 2, 2, 2, 3, 3, 3]) and np.all(o[10:] == -7)
+
+
+def mask_case(seed, n_cont, max_len):
+    rng = np.random.default_rng(seed)
+    lens = rng.integers(0, max_len, size=n_cont)
+    lens[:4] = [0, 1, 15, 17]
+    offs = np.concatenate([[0], np.cumsum(lens)]).astype(np.int64)
+    br = np.array([rng.integers(-1, L + 3) if L > 0 else rng.integers(-1, 3) for L in lens],
+                  dtype=np.int32)
+    valid = (rng.random(int(offs[-1])) < 0.8).astype(np.uint8)
+    return br, offs, valid
+
+
+@pytest.mark.parametrize("seed,n_cont,max_len", [(0, 50, 300), (1, 600, 40), (2, 9, 20000)])
+def test_suffix_mask(hdl, seed, n_cont, max_len):
+    br, offs, valid = mask_case(seed, n_cont, max_len)
+    ref = oracle.suffix_mask(br, offs, valid)
+    ref_nv = oracle.suffix_mask(br, offs, None)
+    tb, to, tv = (torch.from_numpy(x).cuda() for x in (br, offs, valid))
+    m = hdl.hdl_suffix_mask(tb, to, tv)
+    assert np.array_equal(m.cpu().numpy(), ref)
+    m = hdl.hdl_suffix_mask(tb, to, None, mask_len=int(offs[-1]))
+    assert np.array_equal(m.cpu().numpy(), ref_nv)
+
+
+def test_suffix_mask_unaligned_and_offset_range(hdl):
+    """Byte path (mask not 16-byte aligned) and a range that starts and ends
+    mid-buffer: bytes outside the continuations stay untouched."""
+    br, offs, valid = mask_case(3, 40, 200)
+    total = int(offs[-1])
+    shift = 5
+    offs2 = offs + shift
+    buf = torch.full((total + 2 * shift + 1,), 7, dtype=torch.uint8, device="cuda")
+    vbuf = torch.zeros_like(buf)
+    vbuf[shift:shift + total] = torch.from_numpy(valid).cuda()
+    ref = oracle.suffix_mask(br, offs, valid)
+    for base in (0, 1):            # base 1: neither buffer is 16-byte aligned
+        mview = buf[base:]
+        vview = vbuf[base:]
+        buf.fill_(7)
+        o = torch.from_numpy(offs2 - base).cuda()
+        hdl.hdl_suffix_mask(torch.from_numpy(br).cuda(), o, vview, mask=mview)
+        got = buf.cpu().numpy()
+        lo = shift
+        assert np.all(got[:lo] == 7) and np.all(got[lo + total:] == 7)
+        assert np.array_equal(got[lo:lo + total], ref)

@@ -1,0 +1,103 @@
+"""The five workloads (tiny, math, code, agent, roofline sweep) at their full
+sizes, in the launch configuration the bench times.
+
+tiny and math: the oracle scores every token, so log-probs, scores and the
+end-to-end branch sets are compared in full.  code, agent and the sweep: the
+oracle scores sampled tokens one by one (first, last, random), and selection,
+allocation and masks are compared bit-exactly on the device's own scores."""
+import numpy as np
+import pytest
+import torch
+
+import hdl_synth
+import oracle
+from tests.helpers import (assert_logp_close, check_selection_band, oracle_logprobs,
+                           sample_rows, to_f64)
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def hdl():
+    import __graft_entry__
+    __graft_entry__.build()
+    import paper_2609_36864_gb300 as m
+    return m
+
+
+def run_path(hdl, wl):
+    k = wl.spec.k
+    lp0, lp1, delta, ws = hdl.hdl_rescore(wl.h_orig, wl.h_hind, wl.w, wl.targets)
+    bp, ns, bd = hdl.hdl_select_branches(delta, wl.valid, wl.root_offsets, k)
+    cb = hdl.hdl_assign_continuations(ns, bp, wl.conts_per_root,
+                                      n_cont=wl.cont_offsets.numel() - 1)
+    mask = hdl.hdl_suffix_mask(cb, wl.cont_offsets, wl.cont_valid)
+    code, raw = hdl.hdl_device_status(ws)
+    assert code == hdl.HDL_OK, (code, hex(raw))
+    return dict(lp0=lp0.cpu().numpy(), lp1=lp1.cpu().numpy(), delta=delta.cpu().numpy(),
+                bp=bp.cpu().numpy(), ns=ns.cpu().numpy(), bd=bd.cpu().numpy(),
+                cb=cb.cpu().numpy(), mask=mask.cpu().numpy())
+
+
+def check_downstream_exact(wl, out):
+    """Selection / allocation / mask of the oracle on the device's scores."""
+    valid = wl.valid.cpu().numpy()
+    offs = wl.root_offsets.cpu().numpy()
+    d = out["delta"].astype(np.float64)
+    pos, nsel, val = oracle.select_branches(d, valid, offs, wl.spec.k)
+    assert np.array_equal(out["ns"], nsel)
+    assert np.array_equal(out["bp"], pos)
+    assert np.array_equal(out["bd"].astype(np.float64), val, equal_nan=True)
+    cb = oracle.assign_continuations(nsel, pos, wl.conts_per_root.cpu().numpy())
+    assert np.array_equal(out["cb"], cb)
+    m = oracle.suffix_mask(cb, wl.cont_offsets.cpu().numpy(), wl.cont_valid.cpu().numpy())
+    assert np.array_equal(out["mask"], m)
+    # invalid (observation) tokens are never branch points
+    for r in range(len(offs) - 1):
+        for t in out["bp"][r, :out["ns"][r]]:
+            assert valid[offs[r] + t]
+
+
+@pytest.mark.parametrize("name", ["tiny", "math"])
+def test_workload_full_oracle(hdl, name):
+    wl = hdl_synth.generate(hdl_synth.SPECS[name], device="cuda")
+    out = run_path(hdl, wl)
+    W = to_f64(wl.w)
+    y = wl.targets.cpu().numpy()
+    r0 = oracle_logprobs(to_f64(wl.h_orig), W, y)
+    r1 = oracle_logprobs(to_f64(wl.h_hind), W, y)
+    assert_logp_close(out["lp0"], r0, name + " orig")
+    assert_logp_close(out["lp1"], r1, name + " hind")
+    rd = oracle.hindsight_divergence(r1, r0)
+    # |Delta| inherits both contexts' errors
+    err = np.abs(out["delta"] - rd)
+    assert np.all(err <= 2e-3 + 1e-3 * (np.abs(r0) + np.abs(r1))), err.max()
+    check_selection_band(out["bp"], out["ns"], rd, wl.valid.cpu().numpy(),
+                         wl.root_offsets.cpu().numpy(), wl.spec.k)
+    check_downstream_exact(wl, out)
+
+
+SAMPLED = ["code", "agent", ("sweep", 32000, 8192), ("sweep", 256000, 262144),
+           ("sweep", 128256, 131072)]
+
+
+@pytest.mark.parametrize("which", SAMPLED, ids=lambda w: w if isinstance(w, str) else
+                         f"sweep_V{w[1]}_N{w[2]}")
+def test_workload_sampled(hdl, which):
+    spec = (hdl_synth.SPECS[which] if isinstance(which, str)
+            else hdl_synth.sweep_spec(which[1], which[2]))
+    wl = hdl_synth.generate(spec, device="cuda")
+    out = run_path(hdl, wl)
+    rows = sample_rows(wl.n_tokens, 40, seed=spec.d)
+    idx = torch.from_numpy(rows).cuda()
+    W = to_f64(wl.w)
+    y = wl.targets.cpu().numpy()[rows]
+    r0 = oracle.target_logprobs(to_f64(wl.h_orig.index_select(0, idx)), W, y)
+    r1 = oracle.target_logprobs(to_f64(wl.h_hind.index_select(0, idx)), W, y)
+    del W
+    assert_logp_close(out["lp0"][rows], r0, spec.name + " orig")
+    assert_logp_close(out["lp1"][rows], r1, spec.name + " hind")
+    check_downstream_exact(wl, out)
+    # properties that hold at any size
+    assert np.all(out["lp0"] <= 1e-5) and np.all(out["lp1"] <= 1e-5)
+    assert np.all(np.isfinite(out["delta"])) and np.all(out["delta"] >= 0)
