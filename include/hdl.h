@@ -101,6 +101,42 @@ HDL_API hdl_status hdl_rescore(const void* h_orig, const void* h_hind,
                        float* delta, void* workspace, size_t workspace_bytes,
                        void* cuda_stream);
 
+/* Allocation-free variant of hdl_rescore (the paper has no counterpart: this
+ * is an interface convenience).  It is for callers that must not allocate
+ * device memory while they run: plugin "enqueue" callbacks of inference
+ * runtimes, which forbid allocation during enqueue; processes whose device
+ * memory is owned by a pooling allocator, where a cudaMalloc can fail or
+ * fragment the pool; and latency-critical loops, where cudaMalloc/cudaFree
+ * can synchronise the device.  Instead of a caller-provided workspace it uses
+ * one file-scope device array of HDL_STATIC_SCRATCH_BYTES (16 MiB) that every
+ * GPU which loads the library holds until the process exits.  It calls no
+ * cudaMalloc, cudaFree or allocating library routine.
+ *
+ * Arguments and results are those of hdl_rescore, without the workspace.
+ *   - Returns HDL_ERR_UNSUPPORTED, before launching anything, when the
+ *     problem needs more than HDL_STATIC_SCRATCH_BYTES of scratch, i.e. when
+ *     hdl_rescore_workspace_bytes(n_tokens, d, vocab, dt) exceeds it
+ *     (e.g. at vocab = 152064 about 27,000 tokens fit; at vocab = 32000
+ *     about 123,000).
+ *   - The first call on a device looks up the array's device address (with
+ *     that device current) and caches it; make that first call before any
+ *     stream capture.
+ *   - Every call on a device shares the one array and leaves its contents
+ *     behind; each call clears the status word it needs.  Calls that overlap
+ *     on the GPU (e.g. on two streams at once) race on the array: serialise
+ *     them.
+ *   - scratch_out (host pointer, may be NULL) receives the array's device
+ *     address, which hdl_device_status() accepts (with
+ *     HDL_STATIC_SCRATCH_BYTES) to read the device status of the last call. */
+#define HDL_STATIC_SCRATCH_BYTES ((size_t)16 << 20)
+
+HDL_API hdl_status hdl_rescore_noalloc(const void* h_orig, const void* h_hind,
+                               const void* w_lmhead, hdl_dtype dt,
+                               const int32_t* targets, int64_t n_tokens,
+                               int32_t d, int32_t vocab, float* logp_orig,
+                               float* logp_hind, float* delta,
+                               const void** scratch_out, void* cuda_stream);
+
 /* Synchronises `cuda_stream`, then reads the status word of a re-scoring
  * workspace.  Returns HDL_OK, HDL_ERR_TIMEOUT or HDL_ERR_BAD_TARGET (the
  * device condition), or HDL_ERR_CUDA / HDL_ERR_INVALID_ARG for the call

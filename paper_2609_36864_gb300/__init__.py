@@ -20,12 +20,14 @@ __all__ = [
     "HdlError", "lib", "library_path", "HDL_OK", "HDL_BF16", "HDL_F32",
     "hdl_abi_version", "hdl_status_string", "hdl_rescore_workspace_bytes",
     "hdl_rescore", "hdl_device_status", "hdl_select_branches",
-    "hdl_assign_continuations", "hdl_suffix_mask",
+    "hdl_assign_continuations", "hdl_suffix_mask", "hdl_rescore_noalloc",
+    "HDL_STATIC_SCRATCH_BYTES",
 ]
 
 HDL_OK, HDL_ERR_INVALID_ARG, HDL_ERR_UNSUPPORTED, HDL_ERR_WORKSPACE = 0, 1, 2, 3
 HDL_ERR_CUDA, HDL_ERR_TIMEOUT, HDL_ERR_BAD_TARGET = 4, 5, 6
 HDL_BF16, HDL_F32 = 0, 1
+HDL_STATIC_SCRATCH_BYTES = 16 << 20
 
 _PKG = os.path.dirname(os.path.abspath(__file__))
 _lib = None
@@ -67,6 +69,9 @@ def _declare(L):
     L.hdl_assign_continuations.argtypes = [vp, vp, i32, i32, vp, i32, vp, i64, vp]
     L.hdl_suffix_mask.restype = ctypes.c_int
     L.hdl_suffix_mask.argtypes = [vp, vp, i32, vp, vp, i64, vp]
+    L.hdl_rescore_noalloc.restype = ctypes.c_int
+    L.hdl_rescore_noalloc.argtypes = [vp, vp, vp, ctypes.c_int, vp, i64, i32, i32, vp, vp, vp,
+                                      ctypes.POINTER(ctypes.c_void_p), vp]
     return L
 
 
@@ -255,3 +260,30 @@ def hdl_suffix_mask(cont_branch, cont_offsets, cont_valid=None, mask=None,
                                  _ptr(mask), mask.numel(), _stream(stream))
     _check("hdl_suffix_mask", code)
     return mask
+
+
+def hdl_rescore_noalloc(h_orig, h_hind, w_lmhead, targets, logp_orig, logp_hind, delta=None,
+                        stream=None):
+    """hdl_rescore without a workspace, for callers that must not allocate
+    device memory while they run (inference-runtime plugins, pool-owned
+    device memory, latency-critical loops).  Scratch is one static 16 MiB
+    device array shared by all calls: calls that overlap on the GPU race, and
+    problems needing more scratch are rejected (HDL_ERR_UNSUPPORTED).  Every
+    output tensor must be given; nothing is allocated here either.  Returns
+    the device address of the scratch array, which hdl_device_status()
+    accepts."""
+    for t, n in ((h_orig, "h_orig"), (h_hind, "h_hind"), (w_lmhead, "w_lmhead")):
+        _dev(t, n)
+    _dev(targets, "targets", torch.int32)
+    for t, n in ((logp_orig, "logp_orig"), (logp_hind, "logp_hind")):
+        _dev(t, n, torch.float32)
+    if delta is not None:
+        _dev(delta, "delta", torch.float32)
+    N, d = h_orig.shape
+    scratch = ctypes.c_void_p(0)
+    code = lib().hdl_rescore_noalloc(_ptr(h_orig), _ptr(h_hind), _ptr(w_lmhead),
+                                     _hdl_dtype(h_orig), _ptr(targets), N, d,
+                                     w_lmhead.shape[0], _ptr(logp_orig), _ptr(logp_hind),
+                                     _ptr(delta), ctypes.byref(scratch), _stream(stream))
+    _check("hdl_rescore_noalloc", code)
+    return scratch.value

@@ -505,3 +505,49 @@ extern "C" hdl_status hdl_device_status(const void* workspace, size_t workspace_
   if (word & kStatusBadTarget) return HDL_ERR_BAD_TARGET;
   return HDL_OK;
 }
+
+// ---------------------------------------------------------------------------
+// Allocation-free variant: the scratch lives in one file-scope device array.
+// Host code may not use the array's name as a device address (it is a
+// host-side stand-in); its device address is looked up once per device.
+static __device__ __align__(256) uint8_t g_static_scratch[HDL_STATIC_SCRATCH_BYTES];
+
+namespace {
+constexpr int kMaxDevices = 128;
+std::mutex g_scratch_mu;
+void* g_scratch_addr[kMaxDevices] = {};
+
+hdl_status static_scratch_address(void** out) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return HDL_ERR_CUDA;
+  if (dev < 0 || dev >= kMaxDevices) return HDL_ERR_UNSUPPORTED;
+  std::lock_guard<std::mutex> lock(g_scratch_mu);
+  if (g_scratch_addr[dev] == nullptr) {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_static_scratch) != cudaSuccess || p == nullptr)
+      return HDL_ERR_CUDA;
+    g_scratch_addr[dev] = p;
+  }
+  *out = g_scratch_addr[dev];
+  return HDL_OK;
+}
+}  // namespace
+
+extern "C" hdl_status hdl_rescore_noalloc(const void* h_orig, const void* h_hind,
+                                          const void* w_lmhead, hdl_dtype dt,
+                                          const int32_t* targets, int64_t n_tokens, int32_t d,
+                                          int32_t vocab, float* logp_orig, float* logp_hind,
+                                          float* delta, const void** scratch_out,
+                                          void* cuda_stream) {
+  const hdl_status sh = check_shape(n_tokens, d, vocab, dt);
+  if (sh != HDL_OK) return sh;
+  if (n_tokens == 0) return HDL_OK;
+  if (geometry(n_tokens, d, vocab, dt).total > HDL_STATIC_SCRATCH_BYTES)
+    return HDL_ERR_UNSUPPORTED;
+  void* ws = nullptr;
+  const hdl_status st = static_scratch_address(&ws);
+  if (st != HDL_OK) return st;
+  if (scratch_out) *scratch_out = ws;
+  return hdl_rescore(h_orig, h_hind, w_lmhead, dt, targets, n_tokens, d, vocab, logp_orig,
+                     logp_hind, delta, ws, HDL_STATIC_SCRATCH_BYTES, cuda_stream);
+}
