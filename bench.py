@@ -67,6 +67,23 @@ def peaks():
     return 1900.0, 1700.0, 6800.0, "fallback"
 
 
+def committed_traffic(workload: str):
+    """DRAM bytes per launch of the re-scoring kernel from the committed ncu
+    summary, or None if the kernel sources changed since it was taken."""
+    import hashlib
+    prof = os.path.join(ROOT, "profiles", "rescore_lse_traffic.md")
+    csrc = os.path.join(ROOT, "paper_2609_36864_gb300", "csrc")
+    if not os.path.exists(prof):
+        return None
+    h = [hashlib.sha256(open(os.path.join(csrc, f), "rb").read()).hexdigest()[:16]
+         for f in ("rescore.cu", "ptx_sm103.cuh")]
+    for line in open(prof):
+        f = [x.strip() for x in line.strip().strip("|").split("|")]
+        if len(f) >= 5 and f[0] == workload and f[1:3] == h:
+            return float(f[3]) + float(f[4])
+    return None
+
+
 class ClockSampler:
     """nvidia-smi clocks and throttle reasons sampled during the timed region."""
     Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
@@ -363,7 +380,8 @@ def run_gpu(args, world, rank, local):
         "roofline": {"bound": "tensor", "kernel": "rescore_lse_kernel (+ merge)",
                      "achieved": achieved, "peak": sustained, "unit": "TFLOP/s",
                      "frac": achieved / sustained, "peak_kind": f"bf16 sustained ({src})",
-                     "frac_of_burst": achieved / burst, "traffic": None,
+                     "frac_of_burst": achieved / burst,
+                     "traffic": committed_traffic(spec.name),
                      "rescore_ms": rescore_ms},
         "cpu_baseline": cpu, "e2e": e2e, "clocks": clk,
         "gpu_launches": Path.LAUNCHES_PER_STEP * args.steps,
