@@ -31,6 +31,8 @@
 #include <cudaTypedefs.h>
 
 #include <cmath>
+#include <cstdio>
+#include <cstdlib>
 #include <cstdint>
 #include <mutex>
 
@@ -44,17 +46,42 @@ namespace {
 constexpr int kBM = 128;             // rows per tile = TMEM lanes
 constexpr int kBN = 256;             // vocabulary columns per tile
 constexpr int kRowBytes = 128;       // K bytes per stage (one 128-byte swizzle row)
-constexpr int kStages = 4;
 constexpr int kTilesPerChunk = 16;   // 4096 vocabulary entries per unit
-constexpr int kGroupM = 16;          // M-tiles per rasterisation group
+#ifndef HDL_GROUP_M
+#define HDL_GROUP_M 16
+#endif
+#ifndef HDL_MODE
+#define HDL_MODE 1
+#endif
+constexpr int kGroupM = HDL_GROUP_M; // M-tiles per rasterisation group (even)
+constexpr int kMode = HDL_MODE;      // CTA organisation, see Cfg
 constexpr int kThreads = 192;
+static_assert(kGroupM % 2 == 0 && kGroupM >= 2, "group of M-tiles must be even");
+static_assert(kMode >= 0 && kMode <= 3, "mode 0 .. 3");
 constexpr int kAStage = kBM * kRowBytes;        // 16 KiB
-constexpr int kBStage = kBN * kRowBytes;        // 32 KiB
-constexpr int kStageBytes = kAStage + kBStage;  // 48 KiB
 constexpr int kMmaPerStage = kRowBytes / 32;    // 32 bytes of K per MMA
 constexpr int kTmemCols = 2 * kBN;              // two accumulator buffers
-constexpr int kBarOffset = kStages * kStageBytes;
-constexpr int kSmemBytes = kBarOffset + 256 + 1024;   // + barriers + alignment slack
+
+// CTA organisation of the kernel:
+//   mode 0  one CTA per unit, 128 x 256 MMA (cta_group::1), whole W tiles;
+//   mode 1  clusters of two CTAs on neighbouring M-tiles; each loads half of
+//           every W tile and multicasts it into both CTAs (1-CTA MMAs);
+//   mode 2  clusters of two CTAs running the 256 x 256 pair MMA
+//           (cta_group::2): each CTA holds its 128 H rows and one 128-row
+//           half of the W tile, so a stage is 32 KiB and the ring 6 deep;
+//   mode 3  as mode 1 with clusters of four CTAs, each loading a quarter.
+template <int M>
+struct Cfg {
+  static constexpr bool kCluster = M != 0;
+  static constexpr int kCS = M == 3 ? 4 : (M != 0 ? 2 : 1);      // CTAs per cluster
+  static constexpr bool kMulticast = M == 1 || M == 3;            // W parts multicast
+  static constexpr int kBRows = M == 2 ? kBN / 2 : kBN;  // W rows held per CTA
+  static constexpr int kBStage = kBRows * kRowBytes;
+  static constexpr int kStageBytes = kAStage + kBStage;
+  static constexpr int kStages = M == 2 ? 6 : 4;
+  static constexpr int kBarOffset = kStages * kStageBytes;
+  static constexpr int kSmemBytes = kBarOffset + 256 + 1024;  // + barriers + alignment
+};
 constexpr uint64_t kDefaultTimeoutNs = 4000000000ull;   // 4 s per wait
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kLn2 = 0.6931471805599453f;
@@ -68,10 +95,11 @@ struct RescoreArgs {
   int32_t vocab;
   int32_t num_kb;      // K steps (d * esize / 128)
   int32_t num_m_ctx;   // M-tiles per context
-  int32_t num_m;       // M-tiles, both contexts
+  int32_t num_m;       // M-tiles, both contexts (even)
   int32_t num_vt;      // vocabulary tiles
   int32_t num_chunks;
-  int32_t num_units;
+  int32_t num_units;   // work units (per CTA pair in pair mode)
+  int32_t group_m;     // M-tiles per rasterisation group (even)
   uint64_t timeout_ns;
 };
 
@@ -82,16 +110,21 @@ struct Unit {
   int vt0, vt1;  // vocabulary tiles [vt0, vt1)
 };
 
-// Grouped rasterisation: consecutive units run through kGroupM M-tiles
+// Grouped rasterisation: consecutive units run through group_m M-tiles
 // first, then the chunks, so concurrently running units share both their
-// H tiles and their W tiles in L2.
-__device__ __forceinline__ Unit decode_unit(int u, const RescoreArgs& a) {
-  const int per_group = kGroupM * a.num_chunks;
+// H tiles and their W tiles in L2.  In pair mode a unit covers the two
+// M-tiles 2p and 2p+1 (one per CTA of the cluster) over one chunk.
+template <int kCS>
+__device__ __forceinline__ Unit decode_unit(int u, const RescoreArgs& a, int rank) {
+  const int tiles = (a.num_m + kCS - 1) / kCS;   // cluster tiles (last may be partly empty)
+  const int gm = a.group_m / kCS > 0 ? a.group_m / kCS : 1;
+  const int per_group = gm * a.num_chunks;
   const int g = u / per_group;
-  const int first = g * kGroupM;
-  const int gsz = min(a.num_m - first, kGroupM);
+  const int first = g * gm;
+  const int gsz = min(tiles - first, gm);
   const int r = u - g * per_group;
-  const int mt = first + r % gsz;
+  const int t = first + r % gsz;
+  const int mt = kCS * t + rank;   // >= num_m: an empty tile (all rows past the end)
   Unit w;
   w.chunk = r / gsz;
   w.ctx = mt >= a.num_m_ctx ? 1 : 0;
@@ -118,38 +151,50 @@ __device__ __forceinline__ void lse_fold(const float (&x)[32], float& m2, float&
   m2 = m_new;
 }
 
-template <bool kTf32>
+// One persistent kernel for both contexts.  See Cfg for the three CTA
+// organisations.  In the cluster modes a stage may be refilled only once the
+// MMAs of the pair are done with it (mode 1: both CTAs' commits arrive on the
+// stage's empty barrier in both CTAs; mode 2: the even CTA's pair-MMA commit
+// arrives in both), and in mode 2 both CTAs' copies are counted on the even
+// CTA's full barrier and both epilogues release TMEM to the even CTA.
+template <bool kTf32, int M>
 __global__ void __launch_bounds__(kThreads, 1)
     rescore_lse_kernel(const __grid_constant__ CUtensorMap tm_h0,
                        const __grid_constant__ CUtensorMap tm_h1,
                        const __grid_constant__ CUtensorMap tm_w, const RescoreArgs a) {
+  using C = Cfg<M>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>(
       (reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~static_cast<uintptr_t>(1023));
   const uint32_t sbase = smem_addr(smem);
-  const uint32_t sA = sbase;                       // kStages x 16 KiB
-  const uint32_t sB = sbase + kStages * kAStage;   // kStages x 32 KiB
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + kBarOffset);
+  const uint32_t sA = sbase;                          // kStages x 16 KiB
+  const uint32_t sB = sbase + C::kStages * kAStage;   // kStages x kBStage
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + C::kBarOffset);
   const uint32_t bar0 = smem_addr(bars);
   auto full_bar = [&](int s) { return bar0 + 8u * s; };
-  auto empty_bar = [&](int s) { return bar0 + 8u * (kStages + s); };
-  auto tfull_bar = [&](int b) { return bar0 + 8u * (2 * kStages + b); };
-  auto tempty_bar = [&](int b) { return bar0 + 8u * (2 * kStages + 2 + b); };
-  const uint32_t done_bar = bar0 + 8u * (2 * kStages + 4);
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + kBarOffset + 8 * (2 * kStages + 5));
+  auto empty_bar = [&](int s) { return bar0 + 8u * (C::kStages + s); };
+  auto tfull_bar = [&](int b) { return bar0 + 8u * (2 * C::kStages + b); };
+  auto tempty_bar = [&](int b) { return bar0 + 8u * (2 * C::kStages + 2 + b); };
+  const uint32_t done_bar = bar0 + 8u * (2 * C::kStages + 4);
+  uint32_t* tmem_slot =
+      reinterpret_cast<uint32_t*>(smem + C::kBarOffset + 8 * (2 * C::kStages + 5));
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
+  const int rank = C::kCluster ? static_cast<int>(cluster_ctarank()) : 0;
+  const bool leader = rank == 0;
+  const int u_first = C::kCluster ? static_cast<int>(cluster_id_x()) : static_cast<int>(blockIdx.x);
+  const int u_step = C::kCluster ? static_cast<int>(cluster_count_x()) : static_cast<int>(gridDim.x);
 
   if (threadIdx.x == 0) {
-    for (int s = 0; s < kStages; ++s) {
+    for (int s = 0; s < C::kStages; ++s) {
       mbar_init(full_bar(s), 1);
-      mbar_init(empty_bar(s), 1);
+      mbar_init(empty_bar(s), C::kMulticast ? C::kCS : 1);
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(tfull_bar(b), 1);
-      mbar_init(tempty_bar(b), 4);
+      mbar_init(tempty_bar(b), M == 2 ? 8 : 4);
     }
     mbar_init(done_bar, 1);
     *abort_flag = 0;
@@ -160,9 +205,16 @@ __global__ void __launch_bounds__(kThreads, 1)
     tma_prefetch_desc(&tm_h1);
     tma_prefetch_desc(&tm_w);
   }
-  if (warp == 1) tmem_alloc(smem_addr(tmem_slot), kTmemCols);
+  if (warp == 1) {
+    if constexpr (M == 2)
+      tmem_alloc_pair(smem_addr(tmem_slot), kTmemCols);
+    else
+      tmem_alloc(smem_addr(tmem_slot), kTmemCols);
+  }
   tc_fence_before();
   __syncthreads();
+  // the peer's barriers must exist before anything is signalled into them
+  if constexpr (C::kCluster) cluster_sync_all();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
 
@@ -174,8 +226,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       int stage = 0;
       uint32_t phase = 0, pend = 0, pend_par = 0;
       bool ok = true;
-      for (int u = blockIdx.x; ok && u < a.num_units; u += gridDim.x) {
-        const Unit w = decode_unit(u, a);
+      for (int u = u_first; ok && u < a.num_units; u += u_step) {
+        const Unit w = decode_unit<C::kCS>(u, a, rank);
         const CUtensorMap* tmA = w.ctx ? &tm_h1 : &tm_h0;
         for (int vt = w.vt0; ok && vt < w.vt1; ++vt) {
           for (int kb = 0; kb < a.num_kb; ++kb) {
@@ -183,13 +235,28 @@ __global__ void __launch_bounds__(kThreads, 1)
               ok = false;
               break;
             }
-            mbar_arrive_expect_tx(full_bar(stage), kStageBytes);
             const int32_t kx = kb * (kRowBytes / (kTf32 ? 4 : 2));
-            tma_load_2d(sA + stage * kAStage, tmA, kx, w.row0, full_bar(stage));
-            tma_load_2d(sB + stage * kBStage, &tm_w, kx, vt * kBN, full_bar(stage));
+            const uint32_t dA = sA + stage * kAStage, dB = sB + stage * C::kBStage;
+            if constexpr (M == 2) {
+              const uint32_t fb = mapa_shared(full_bar(stage), 0);
+              if (leader) mbar_arrive_expect_tx(full_bar(stage), 2 * C::kStageBytes);
+              tma_load_2d_pair(dA, tmA, kx, w.row0, fb);
+              tma_load_2d_pair(dB, &tm_w, kx, vt * kBN + rank * (kBN / 2), fb);
+            } else if constexpr (C::kMulticast) {
+              constexpr int part = kBN / C::kCS;   // W rows this CTA fetches
+              mbar_arrive_expect_tx(full_bar(stage), C::kStageBytes);
+              tma_load_2d(dA, tmA, kx, w.row0, full_bar(stage));
+              tma_load_2d_multicast(dB + static_cast<uint32_t>(rank * part * kRowBytes), &tm_w,
+                                    kx, vt * kBN + rank * part, full_bar(stage),
+                                    static_cast<uint16_t>((1u << C::kCS) - 1u));
+            } else {
+              mbar_arrive_expect_tx(full_bar(stage), C::kStageBytes);
+              tma_load_2d(dA, tmA, kx, w.row0, full_bar(stage));
+              tma_load_2d(dB, &tm_w, kx, vt * kBN, full_bar(stage));
+            }
             pend |= 1u << stage;
             pend_par = (pend_par & ~(1u << stage)) | (phase << stage);
-            if (++stage == kStages) {
+            if (++stage == C::kStages) {
               stage = 0;
               phase ^= 1u;
             }
@@ -198,20 +265,29 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       if (!ok) {
         // Aborted: let the copies already issued land before the CTA exits.
-        for (int s = 0; s < kStages; ++s)
-          if ((pend >> s) & 1u) mbar_wait_drain(full_bar(s), (pend_par >> s) & 1u, 100000000ull);
+        if (M == 2 && !leader) {
+          // this CTA's copies are counted on the even CTA's barriers: wait a
+          // bounded 2 ms, far longer than a copy takes
+          const uint64_t t0 = global_timer_ns();
+          while (global_timer_ns() - t0 < 2000000ull) {
+          }
+        } else {
+          for (int s = 0; s < C::kStages; ++s)
+            if ((pend >> s) & 1u)
+              mbar_wait_drain(full_bar(s), (pend_par >> s) & 1u, 100000000ull);
+        }
       }
     }
     __syncwarp();
   } else if (warp == 1) {
     // --------------------------------------------------------- MMA issuer
-    if (lane == 0) {
-      constexpr uint32_t idesc = make_idesc(kTf32 ? 2u : 1u, kBM, kBN);
+    if (lane == 0 && (M != 2 || leader)) {
+      constexpr uint32_t idesc = make_idesc(kTf32 ? 2u : 1u, M == 2 ? 2 * kBM : kBM, kBN);
       int stage = 0;
       uint32_t phase = 0, tile = 0;
       bool ok = true;
-      for (int u = blockIdx.x; ok && u < a.num_units; u += gridDim.x) {
-        const Unit w = decode_unit(u, a);
+      for (int u = u_first; ok && u < a.num_units; u += u_step) {
+        const Unit w = decode_unit<C::kCS>(u, a, rank);
         for (int vt = w.vt0; ok && vt < w.vt1; ++vt, ++tile) {
           const uint32_t buf = tile & 1u, use = (tile >> 1) & 1u;
           if (!mbar_wait_bounded(tempty_bar(buf), use ^ 1u, ctl, kRoleMma)) {
@@ -227,23 +303,42 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
             tc_fence_after();
             const uint32_t a_addr = sA + stage * kAStage;
-            const uint32_t b_addr = sB + stage * kBStage;
+            const uint32_t b_addr = sB + stage * C::kBStage;
 #pragma unroll
-            for (int kk = 0; kk < kMmaPerStage; ++kk)
-              tc_mma<kTf32>(d_tmem, smem_desc_sw128(a_addr + 32 * kk),
-                            smem_desc_sw128(b_addr + 32 * kk), idesc,
-                            (kb | kk) != 0 ? 1u : 0u);
-            tc_commit(empty_bar(stage));
-            if (++stage == kStages) {
+            for (int kk = 0; kk < kMmaPerStage; ++kk) {
+              const uint64_t ad = smem_desc_sw128(a_addr + 32 * kk);
+              const uint64_t bd = smem_desc_sw128(b_addr + 32 * kk);
+              const uint32_t acc = (kb | kk) != 0 ? 1u : 0u;
+              if constexpr (M == 2)
+                tc_mma_pair<kTf32>(d_tmem, ad, bd, idesc, acc);
+              else
+                tc_mma<kTf32>(d_tmem, ad, bd, idesc, acc);
+            }
+            if constexpr (M == 2)
+              tc_commit_pair_multicast(empty_bar(stage), 0x3);
+            else if constexpr (C::kMulticast)
+              tc_commit_multicast(empty_bar(stage), static_cast<uint16_t>((1u << C::kCS) - 1u));
+            else
+              tc_commit(empty_bar(stage));
+            if (++stage == C::kStages) {
               stage = 0;
               phase ^= 1u;
             }
           }
-          if (ok) tc_commit(tfull_bar(buf));
+          if (ok) {
+            if constexpr (M == 2)
+              tc_commit_pair_multicast(tfull_bar(buf), 0x3);
+            else
+              tc_commit(tfull_bar(buf));
+          }
         }
       }
-      // Every MMA issued above must finish before TMEM is released.
-      tc_commit(done_bar);
+      // Every MMA issued above (and the arrivals it feeds) must finish before
+      // TMEM is released and before the peer CTA may exit.
+      if constexpr (M == 2)
+        tc_commit_pair(done_bar);
+      else
+        tc_commit(done_bar);
       mbar_wait_drain(done_bar, 0, 1000000000ull);
     }
     __syncwarp();
@@ -254,8 +349,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t lane_addr = static_cast<uint32_t>(q * 32) << 16;
     uint32_t tile = 0;
     bool ok = true;
-    for (int u = blockIdx.x; ok && u < a.num_units; u += gridDim.x) {
-      const Unit w = decode_unit(u, a);
+    for (int u = u_first; ok && u < a.num_units; u += u_step) {
+      const Unit w = decode_unit<C::kCS>(u, a, rank);
       const int64_t row = static_cast<int64_t>(w.row0) + r_in_tile;
       const bool in_range = row < a.n_tokens;
       const int32_t y = in_range ? __ldg(a.targets + row) : -1;
@@ -295,7 +390,12 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         tc_fence_before();
         __syncwarp();
-        if (lane == 0) mbar_arrive(tempty_bar(buf));
+        if (lane == 0) {
+          if constexpr (M == 2)
+            mbar_arrive_cluster(mapa_shared(tempty_bar(buf), 0));
+          else
+            mbar_arrive(tempty_bar(buf));
+        }
       }
       if (ok && in_range) {
         const int64_t rows_total = 2 * a.n_tokens;
@@ -308,9 +408,15 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   tc_fence_before();
   __syncthreads();
+  // neither CTA of a pair may leave while the other can still write into
+  // its shared memory or TMEM or arrive on its barriers
+  if constexpr (C::kCluster) cluster_sync_all();
   if (warp == 1) {
     tc_fence_after();
-    tmem_dealloc(tmem_base, kTmemCols);
+    if constexpr (M == 2)
+      tmem_dealloc_pair(tmem_base, kTmemCols);
+    else
+      tmem_dealloc(tmem_base, kTmemCols);
   }
 }
 
@@ -405,6 +511,48 @@ bool make_operand_map(CUtensorMap* m, const void* ptr, int64_t rows, int32_t d, 
   return r == CUDA_SUCCESS;
 }
 
+// One persistent CTA per SM (cluster modes: as many clusters of two as can
+// be resident at once).
+template <bool kTf32, int M>
+hdl_status launch_rescore(const CUtensorMap& tm_h0, const CUtensorMap& tm_h1,
+                          const CUtensorMap& tm_w, const RescoreArgs& a, int sms,
+                          cudaStream_t st) {
+  using C = Cfg<M>;
+  auto kern = rescore_lse_kernel<kTf32, M>;
+  if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes) !=
+      cudaSuccess)
+    return HDL_ERR_CUDA;
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute attr[1];
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = C::kSmemBytes;
+  cfg.stream = st;
+  if (C::kCluster) {
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = C::kCS;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    int64_t clusters = sms / C::kCS;
+    cfg.gridDim = dim3(static_cast<unsigned>(C::kCS * clusters));
+    int resident = 0;
+    if (cudaOccupancyMaxActiveClusters(&resident, kern, &cfg) == cudaSuccess && resident > 0 &&
+        resident < clusters)
+      clusters = resident;
+    if (clusters > a.num_units) clusters = a.num_units;
+    if (clusters < 1) clusters = 1;
+    cfg.gridDim = dim3(static_cast<unsigned>(C::kCS * clusters));
+    if (std::getenv("HDL_PRINT_GRID"))
+      std::fprintf(stderr, "hdl: mode %d grid %u (%lld clusters of %d, %d resident)\n", M,
+                   cfg.gridDim.x, static_cast<long long>(clusters), C::kCS, resident);
+  } else {
+    cfg.gridDim = dim3(static_cast<unsigned>(a.num_units < sms ? a.num_units : sms));
+  }
+  if (cudaLaunchKernelEx(&cfg, kern, tm_h0, tm_h1, tm_w, a) != cudaSuccess) return HDL_ERR_CUDA;
+  return HDL_OK;
+}
+
 hdl_status check_shape(int64_t n_tokens, int32_t d, int32_t vocab, hdl_dtype dt) {
   if (n_tokens < 0 || d <= 0 || vocab <= 0) return HDL_ERR_INVALID_ARG;
   if (dt != HDL_BF16 && dt != HDL_F32) return HDL_ERR_INVALID_ARG;
@@ -447,7 +595,7 @@ extern "C" hdl_status hdl_rescore(const void* h_orig, const void* h_hind, const 
   CUtensorMap tm_h0, tm_h1, tm_w;
   if (!make_operand_map(&tm_h0, h_orig, n_tokens, d, g.esize, kBM) ||
       !make_operand_map(&tm_h1, h_hind, n_tokens, d, g.esize, kBM) ||
-      !make_operand_map(&tm_w, w_lmhead, vocab, d, g.esize, kBN))
+      !make_operand_map(&tm_w, w_lmhead, vocab, d, g.esize, kBN / Cfg<kMode>::kCS))
     return HDL_ERR_CUDA;
 
   uint8_t* ws = static_cast<uint8_t*>(workspace);
@@ -463,7 +611,8 @@ extern "C" hdl_status hdl_rescore(const void* h_orig, const void* h_hind, const 
   a.num_m = g.num_m;
   a.num_vt = g.num_vt;
   a.num_chunks = g.num_chunks;
-  a.num_units = static_cast<int32_t>(g.num_units);
+  a.num_units = static_cast<int32_t>(ceil_div(g.num_m, Cfg<kMode>::kCS) * g.num_chunks);
+  a.group_m = kGroupM;
   a.timeout_ns = kDefaultTimeoutNs;
 
   cudaStream_t st = as_stream(cuda_stream);
@@ -471,18 +620,10 @@ extern "C" hdl_status hdl_rescore(const void* h_orig, const void* h_hind, const 
 
   const int sms = current_sm_count();
   if (sms <= 0) return HDL_ERR_CUDA;
-  const int grid = static_cast<int>(g.num_units < sms ? g.num_units : sms);
-  if (dt == HDL_F32) {
-    if (cudaFuncSetAttribute(rescore_lse_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             kSmemBytes) != cudaSuccess)
-      return HDL_ERR_CUDA;
-    rescore_lse_kernel<true><<<grid, kThreads, kSmemBytes, st>>>(tm_h0, tm_h1, tm_w, a);
-  } else {
-    if (cudaFuncSetAttribute(rescore_lse_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             kSmemBytes) != cudaSuccess)
-      return HDL_ERR_CUDA;
-    rescore_lse_kernel<false><<<grid, kThreads, kSmemBytes, st>>>(tm_h0, tm_h1, tm_w, a);
-  }
+  const hdl_status ls =
+      dt == HDL_F32 ? launch_rescore<true, kMode>(tm_h0, tm_h1, tm_w, a, sms, st)
+                    : launch_rescore<false, kMode>(tm_h0, tm_h1, tm_w, a, sms, st);
+  if (ls != HDL_OK) return ls;
   if (launch_status() != HDL_OK) return HDL_ERR_CUDA;
 
   const int64_t mblocks = ceil_div(n_tokens, 256);
