@@ -11,6 +11,9 @@ Functions and the passages they follow (arXiv 2609.36864):
                          under a softmax over the vocabulary at temperature 1
                          (the rollout temperature of Section 4.1).
   hindsight_divergence   Section 3.2, Eq. (div): s_i = |log p^H_i(y_i) - log p^0_i(y_i)|.
+  next_token_entropy     Section 4.1 "Rollout protocols", the Entropy selector:
+                         the entropy of the next-token distribution under the
+                         original context, H = -sum_v p_v log p_v.
   select_branches        Section 3.2 (rank the candidate positions of a root by
                          s_i, take the highest), candidates = policy-generated
                          tokens (Section 3.1); optional spacing rule of
@@ -50,7 +53,8 @@ import math
 import numpy as np
 
 __all__ = [
-    "widen", "target_logprobs", "hindsight_divergence", "select_branches",
+    "widen", "target_logprobs", "hindsight_divergence", "next_token_entropy",
+    "select_branches",
     "allocate_counts", "assign_continuations", "suffix_mask",
 ]
 
@@ -94,6 +98,20 @@ def target_logprobs(h: np.ndarray, w: np.ndarray, targets: np.ndarray) -> np.nda
 def hindsight_divergence(logp_hind: np.ndarray, logp_orig: np.ndarray) -> np.ndarray:
     """s_t = |log p^H_t(y_t) - log p^0_t(y_t)| (Eq. div, Section 3.2)."""
     return np.abs(np.asarray(logp_hind, np.float64) - np.asarray(logp_orig, np.float64))
+
+
+def next_token_entropy(h: np.ndarray, w: np.ndarray) -> np.ndarray:
+    """H_t = -sum_v p_v log p_v of p = softmax(h_t W^T), in nats (Section 4.1,
+    the Entropy baseline's ranking signal).  log p_v is formed as
+    z_v - max - log sum exp(z - max), so p_v = 0 contributes 0."""
+    h = np.asarray(h, dtype=np.float64)
+    w = np.asarray(w, dtype=np.float64)
+    if h.shape[0] == 0:
+        return np.zeros(0)
+    z = h @ w.T
+    m = z.max(axis=1, keepdims=True)
+    logp = z - m - np.log(np.exp(z - m).sum(axis=1, keepdims=True))
+    return -(np.exp(logp) * logp).sum(axis=1)
 
 
 def _too_close(t: int, accepted: list, min_gap: int) -> bool:

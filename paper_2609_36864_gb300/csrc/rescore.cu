@@ -9,7 +9,7 @@
 // the tile that holds it.
 //
 // Work unit = (M-tile of 128 rows of one context, vocabulary chunk of
-// kTilesPerChunk 256-wide tiles).  Each unit writes one partial (max, sum)
+// up to 16 256-wide tiles).  Each unit writes one partial (max, sum)
 // per row; a second, tiny kernel merges the chunks, forms both log-probs and
 // |Delta|.  Splitting the vocabulary keeps the set of tiles that the ~150
 // concurrently running units touch small enough to stay in L2 (grouped
@@ -46,18 +46,15 @@ namespace {
 constexpr int kBM = 128;             // rows per tile = TMEM lanes
 constexpr int kBN = 256;             // vocabulary columns per tile
 constexpr int kRowBytes = 128;       // K bytes per stage (one 128-byte swizzle row)
-constexpr int kTilesPerChunk = 16;   // 4096 vocabulary entries per unit
+constexpr int kMaxTilesPerChunk = 16;  // up to 4096 vocabulary entries per unit
+constexpr int64_t kMinUnits = 1216;     // 8 x 152: chunks shrink until this many units
 #ifndef HDL_GROUP_M
 #define HDL_GROUP_M 16
 #endif
-#ifndef HDL_MODE
-#define HDL_MODE 1
-#endif
 constexpr int kGroupM = HDL_GROUP_M; // M-tiles per rasterisation group (even)
-constexpr int kMode = HDL_MODE;      // CTA organisation, see Cfg
+constexpr int kDefaultMode = 1;      // CTA organisation, see Cfg
 constexpr int kThreads = 192;
 static_assert(kGroupM % 2 == 0 && kGroupM >= 2, "group of M-tiles must be even");
-static_assert(kMode >= 0 && kMode <= 3, "mode 0 .. 3");
 constexpr int kAStage = kBM * kRowBytes;        // 16 KiB
 constexpr int kMmaPerStage = kRowBytes / 32;    // 32 bytes of K per MMA
 constexpr int kTmemCols = 2 * kBN;              // two accumulator buffers
@@ -68,13 +65,14 @@ constexpr int kTmemCols = 2 * kBN;              // two accumulator buffers
 //           every W tile and multicasts it into both CTAs (1-CTA MMAs);
 //   mode 2  clusters of two CTAs running the 256 x 256 pair MMA
 //           (cta_group::2): each CTA holds its 128 H rows and one 128-row
-//           half of the W tile, so a stage is 32 KiB and the ring 6 deep;
-//   mode 3  as mode 1 with clusters of four CTAs, each loading a quarter.
+//           half of the W tile, so a stage is 32 KiB and the ring 6 deep.
+// (Clusters of four were measured too: only 36 fit at once, leaving 8 SMs
+// idle, and they were not faster.)
 template <int M>
 struct Cfg {
   static constexpr bool kCluster = M != 0;
-  static constexpr int kCS = M == 3 ? 4 : (M != 0 ? 2 : 1);      // CTAs per cluster
-  static constexpr bool kMulticast = M == 1 || M == 3;            // W parts multicast
+  static constexpr int kCS = M != 0 ? 2 : 1;    // CTAs per cluster
+  static constexpr bool kMulticast = M == 1;     // W halves multicast
   static constexpr int kBRows = M == 2 ? kBN / 2 : kBN;  // W rows held per CTA
   static constexpr int kBStage = kBRows * kRowBytes;
   static constexpr int kStageBytes = kAStage + kBStage;
@@ -98,7 +96,8 @@ struct RescoreArgs {
   int32_t num_m;       // M-tiles, both contexts (even)
   int32_t num_vt;      // vocabulary tiles
   int32_t num_chunks;
-  int32_t num_units;   // work units (per CTA pair in pair mode)
+  int32_t tiles_per_chunk;
+  int32_t num_units;   // work units (per cluster in the cluster modes)
   int32_t group_m;     // M-tiles per rasterisation group (even)
   uint64_t timeout_ns;
 };
@@ -129,8 +128,8 @@ __device__ __forceinline__ Unit decode_unit(int u, const RescoreArgs& a, int ran
   w.chunk = r / gsz;
   w.ctx = mt >= a.num_m_ctx ? 1 : 0;
   w.row0 = (mt - w.ctx * a.num_m_ctx) * kBM;
-  w.vt0 = w.chunk * kTilesPerChunk;
-  w.vt1 = min(w.vt0 + kTilesPerChunk, a.num_vt);
+  w.vt0 = w.chunk * a.tiles_per_chunk;
+  w.vt1 = min(w.vt0 + a.tiles_per_chunk, a.num_vt);
   return w;
 }
 
@@ -458,7 +457,7 @@ __global__ void __launch_bounds__(256)
 struct Geometry {
   int64_t n;
   int esize;
-  int num_kb, num_m_ctx, num_m, num_vt, num_chunks;
+  int num_kb, num_m_ctx, num_m, num_vt, num_chunks, tiles_per_chunk;
   int64_t num_units;
   size_t zt_off, part_off, total;
 };
@@ -471,7 +470,12 @@ Geometry geometry(int64_t n, int32_t d, int32_t vocab, hdl_dtype dt) {
   g.num_m_ctx = static_cast<int>(ceil_div(n, kBM));
   g.num_m = 2 * g.num_m_ctx;
   g.num_vt = static_cast<int>(ceil_div(vocab, kBN));
-  g.num_chunks = static_cast<int>(ceil_div(g.num_vt, kTilesPerChunk));
+  // Small problems split the vocabulary finer so that every SM gets work.
+  g.tiles_per_chunk = kMaxTilesPerChunk;
+  while (g.tiles_per_chunk > 1 &&
+         static_cast<int64_t>(g.num_m) * ceil_div(g.num_vt, g.tiles_per_chunk) < kMinUnits)
+    g.tiles_per_chunk /= 2;
+  g.num_chunks = static_cast<int>(ceil_div(g.num_vt, g.tiles_per_chunk));
   g.num_units = static_cast<int64_t>(g.num_m) * g.num_chunks;
   g.zt_off = 256;
   g.part_off = g.zt_off + align_up(static_cast<size_t>(2 * n) * sizeof(float), 256);
@@ -553,6 +557,18 @@ hdl_status launch_rescore(const CUtensorMap& tm_h0, const CUtensorMap& tm_h1,
   return HDL_OK;
 }
 
+// CTA organisation (see Cfg): kDefaultMode unless HDL_RESCORE_MODE = 0, 1 or
+// 2 is set in the environment (a tuning override; every mode gives the same
+// results bit for bit).
+int rescore_mode() {
+  static const int mode = [] {
+    const char* e = std::getenv("HDL_RESCORE_MODE");
+    if (e && (e[0] == '0' || e[0] == '1' || e[0] == '2') && e[1] == '\0') return e[0] - '0';
+    return kDefaultMode;
+  }();
+  return mode;
+}
+
 hdl_status check_shape(int64_t n_tokens, int32_t d, int32_t vocab, hdl_dtype dt) {
   if (n_tokens < 0 || d <= 0 || vocab <= 0) return HDL_ERR_INVALID_ARG;
   if (dt != HDL_BF16 && dt != HDL_F32) return HDL_ERR_INVALID_ARG;
@@ -592,10 +608,12 @@ extern "C" hdl_status hdl_rescore(const void* h_orig, const void* h_hind, const 
   if (!workspace || !aligned_to(workspace, 256) || workspace_bytes < g.total)
     return HDL_ERR_WORKSPACE;
 
+  const int mode = rescore_mode();
+  const int cs = mode == 0 ? 1 : 2;   // CTAs per cluster
   CUtensorMap tm_h0, tm_h1, tm_w;
   if (!make_operand_map(&tm_h0, h_orig, n_tokens, d, g.esize, kBM) ||
       !make_operand_map(&tm_h1, h_hind, n_tokens, d, g.esize, kBM) ||
-      !make_operand_map(&tm_w, w_lmhead, vocab, d, g.esize, kBN / Cfg<kMode>::kCS))
+      !make_operand_map(&tm_w, w_lmhead, vocab, d, g.esize, kBN / cs))
     return HDL_ERR_CUDA;
 
   uint8_t* ws = static_cast<uint8_t*>(workspace);
@@ -611,7 +629,8 @@ extern "C" hdl_status hdl_rescore(const void* h_orig, const void* h_hind, const 
   a.num_m = g.num_m;
   a.num_vt = g.num_vt;
   a.num_chunks = g.num_chunks;
-  a.num_units = static_cast<int32_t>(ceil_div(g.num_m, Cfg<kMode>::kCS) * g.num_chunks);
+  a.tiles_per_chunk = g.tiles_per_chunk;
+  a.num_units = static_cast<int32_t>(ceil_div(g.num_m, cs) * g.num_chunks);
   a.group_m = kGroupM;
   a.timeout_ns = kDefaultTimeoutNs;
 
@@ -620,9 +639,17 @@ extern "C" hdl_status hdl_rescore(const void* h_orig, const void* h_hind, const 
 
   const int sms = current_sm_count();
   if (sms <= 0) return HDL_ERR_CUDA;
-  const hdl_status ls =
-      dt == HDL_F32 ? launch_rescore<true, kMode>(tm_h0, tm_h1, tm_w, a, sms, st)
-                    : launch_rescore<false, kMode>(tm_h0, tm_h1, tm_w, a, sms, st);
+  const bool tf32 = dt == HDL_F32;
+  hdl_status ls;
+  if (mode == 0)
+    ls = tf32 ? launch_rescore<true, 0>(tm_h0, tm_h1, tm_w, a, sms, st)
+              : launch_rescore<false, 0>(tm_h0, tm_h1, tm_w, a, sms, st);
+  else if (mode == 2)
+    ls = tf32 ? launch_rescore<true, 2>(tm_h0, tm_h1, tm_w, a, sms, st)
+              : launch_rescore<false, 2>(tm_h0, tm_h1, tm_w, a, sms, st);
+  else
+    ls = tf32 ? launch_rescore<true, 1>(tm_h0, tm_h1, tm_w, a, sms, st)
+              : launch_rescore<false, 1>(tm_h0, tm_h1, tm_w, a, sms, st);
   if (ls != HDL_OK) return ls;
   if (launch_status() != HDL_OK) return HDL_ERR_CUDA;
 

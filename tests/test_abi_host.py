@@ -54,14 +54,20 @@ def test_abi_version_and_names(L):
 
 
 def _ws_formula(n, d, V):
-    chunks = -(-(-(-V // 256)) // 16)
-    zt = -(-(2 * n * 4) // 256) * 256
+    """status (256 B) + target logits + per-(chunk, row) partials; the chunk
+    shrinks from 16 vocabulary tiles until there are >= 1216 work units."""
+    cdiv = lambda a, b: -(-a // b)
+    num_m, nvt, tpc = 2 * cdiv(n, 128), cdiv(V, 256), 16
+    while tpc > 1 and num_m * cdiv(nvt, tpc) < 1216:
+        tpc //= 2
+    chunks = cdiv(nvt, tpc)
+    zt = cdiv(2 * n * 4, 256) * 256
     return 256 + zt + chunks * 2 * n * 8
 
 
 @pytest.mark.parametrize("n,d,V", [(0, 64, 1), (1, 64, 1), (2048, 256, 4096),
                                    (18000, 2048, 32000), (327680, 5120, 152064),
-                                   (5, 128, 4097)])
+                                   (5, 128, 4097), (8192, 4096, 32000), (1000, 64, 152064)])
 def test_workspace_bytes(L, n, d, V):
     import paper_2609_36864_gb300 as hdl
     assert hdl.hdl_rescore_workspace_bytes(n, d, V, hdl.HDL_BF16) == _ws_formula(n, d, V)

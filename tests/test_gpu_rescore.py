@@ -111,3 +111,45 @@ def test_rescore_outputs_independent_of_stream_and_repeat(hdl):
     s.synchronize()
     for x, y in zip(a[:3], b[:3]):
         assert torch.equal(x, y)
+
+
+_MODE_SCRIPT = r"""
+import sys, numpy as np, torch
+sys.path.insert(0, sys.argv[1])
+import hdl_synth, paper_2609_36864_gb300 as hdl
+for i, (n, d, V, dt) in enumerate([(700, 256, 9000, "bf16"), (300, 128, 4097, "f32"),
+                                   (5, 64, 300, "bf16")]):
+    spec = hdl_synth.small_spec("modes", n_roots=1, t_lo=n, t_hi=n, d=d, vocab=V, dtype=dt,
+                                seed=40 + i)
+    wl = hdl_synth.generate(spec, device="cuda")
+    lp0, lp1, delta, ws = hdl.hdl_rescore(wl.h_orig, wl.h_hind, wl.w, wl.targets)
+    assert hdl.hdl_device_status(ws)[0] == hdl.HDL_OK
+    np.save(sys.argv[2] + f"_{i}.npy", torch.stack([lp0, lp1, delta]).cpu().numpy())
+"""
+
+
+def test_rescore_cta_modes_agree_bitwise(hdl, tmp_path):
+    """The three CTA organisations of the kernel (single CTA, multicast pair,
+    cta_group::2 pair) give bit-identical results, equal to the oracle's."""
+    import os
+    import subprocess
+    import sys
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    outs = {}
+    for mode in ("0", "1", "2"):
+        env = dict(os.environ, HDL_RESCORE_MODE=mode)
+        stem = str(tmp_path / f"m{mode}")
+        subprocess.run([sys.executable, "-c", _MODE_SCRIPT, root, stem], env=env, check=True,
+                       timeout=300)
+        outs[mode] = [np.load(stem + f"_{i}.npy") for i in range(3)]
+    for i in range(3):
+        assert np.array_equal(outs["0"][i], outs["1"][i], equal_nan=True)
+        assert np.array_equal(outs["0"][i], outs["2"][i], equal_nan=True)
+    # and the shared result is the oracle's (first shape)
+    spec = hdl_synth.small_spec("modes", n_roots=1, t_lo=700, t_hi=700, d=256, vocab=9000,
+                                dtype="bf16", seed=40)
+    wl = hdl_synth.generate(spec, device="cuda")
+    W = to_f64(wl.w)
+    y = wl.targets.cpu().numpy()
+    assert_logp_close(outs["0"][0][0], oracle_logprobs(to_f64(wl.h_orig), W, y), "modes orig")
+    assert_logp_close(outs["0"][0][1], oracle_logprobs(to_f64(wl.h_hind), W, y), "modes hind")

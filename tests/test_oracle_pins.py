@@ -144,6 +144,64 @@ def test_divergence():
     check_divergence(O.hindsight_divergence)
 
 
+# ------------------------------------------------------------------ entropy
+def brute_entropy(h, w):
+    z = [math.fsum(a * b for a, b in zip(h, wv)) for wv in w]
+    den = math.fsum(math.exp(v) for v in z)
+    p = [math.exp(v) / den for v in z]
+    return -math.fsum(q * math.log(q) for q in p if q > 0)
+
+
+def check_entropy(fn):
+    rng = np.random.default_rng(13)
+    for d, V in [(1, 1), (1, 2), (3, 5), (4, 8)]:
+        h = rng.normal(size=(5, d))
+        w = rng.normal(size=(V, d))
+        got = fn(h, w)
+        ref = [brute_entropy(h[i], w) for i in range(5)]
+        assert np.allclose(got, ref, rtol=0, atol=1e-12), (d, V, got, ref)
+    # uniform logits: ln V; V = 1: 0
+    for V in (1, 2, 7, 4096):
+        assert np.allclose(fn(np.ones((2, 3)), np.zeros((V, 3))), math.log(V), atol=1e-13)
+    # two words: the binary entropy of sigmoid(z0 - z1)
+    a, b0, b1 = 0.7, 2.0, -1.0
+    p0 = 1.0 / (1.0 + math.exp(a * b1 - a * b0))
+    hb = -p0 * math.log(p0) - (1 - p0) * math.log(1 - p0)
+    assert abs(fn(np.array([[a]]), np.array([[b0], [b1]]))[0] - hb) < 1e-15
+    # one dominant word: ~0; bounds 0 <= H <= ln V; shift and permutation invariance
+    w = np.zeros((50, 2))
+    w[3, 0] = 60.0
+    assert 0 <= fn(np.array([[1.0, 0.0]]), w)[0] < 1e-20
+    h = rng.normal(size=(6, 8))
+    w = rng.normal(size=(40, 8))
+    H = fn(h, w)
+    assert np.all(H >= 0) and np.all(H <= math.log(40) + 1e-12)
+    h2 = np.concatenate([h, np.ones((6, 1))], axis=1)
+    w2 = np.concatenate([w, np.full((40, 1), 700.0)], axis=1)
+    assert np.allclose(fn(h2, w2), H, atol=1e-10)
+    assert np.allclose(fn(h, w[rng.permutation(40)]), H, atol=1e-12)
+
+
+def test_entropy():
+    check_entropy(O.next_token_entropy)
+
+
+def test_planted_mistakes_entropy():
+    def no_minus(h, w):
+        return -O.next_token_entropy(h, w)
+
+    def log2_units(h, w):
+        return O.next_token_entropy(h, w) / math.log(2)
+
+    def unnormalised(h, w):
+        z = np.asarray(h, float) @ np.asarray(w, float).T
+        e = np.exp(z - z.max(1, keepdims=True))
+        return -(e * np.log(e)).sum(1)
+    for mutant in (no_minus, log2_units, unnormalised):
+        with pytest.raises(AssertionError):
+            check_entropy(mutant)
+
+
 # ----------------------------------------------------------------- selection
 def _beats(delta, a, b):
     return delta[a] > delta[b] or (delta[a] == delta[b] and a < b)
