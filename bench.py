@@ -323,39 +323,66 @@ def run_gpu(args, world, rank, local):
     rescore_ms = float(np.mean([a.elapsed_time(b_) for a, b_ in ev]))
     value = world * N * args.steps / (total_ms / 1e3)
 
-    # ---- end to end: host inputs copied in, results copied out, every step
+    # ---- end to end: every step's inputs are copied host -> device from
+    # pinned memory and its results device -> host.  Inputs are double
+    # buffered: the copy of step i+1 runs on a copy stream while step i
+    # computes (event-ordered), as a serving loop would run it.
     e2e = None
     if not args.no_e2e:
-        host_in = {k: getattr(wl, k).cpu().pin_memory() for k in
-                   ("h_orig", "h_hind", "targets", "valid", "root_offsets", "conts_per_root",
-                    "cont_offsets", "cont_valid")}
-        outs = (path.bp, path.ns, path.bd, path.mask)
-        host_out = [torch.empty(t.shape, dtype=t.dtype, pin_memory=True) for t in outs]
+        import dataclasses
+        keys = ("h_orig", "h_hind", "targets", "valid", "root_offsets", "conts_per_root",
+                "cont_offsets", "cont_valid")
+        host_in = {k: getattr(wl, k).cpu().pin_memory() for k in keys}
+        wl2 = dataclasses.replace(wl, **{k: torch.empty_like(getattr(wl, k)) for k in keys})
+        sets = [(wl, path), (wl2, Path(hdl, wl2))]
+        host_out = [[torch.empty(t.shape, dtype=t.dtype, pin_memory=True)
+                     for t in (p_.bp, p_.ns, p_.bd, p_.mask)] for _, p_ in sets]
         h2d = sum(t.numel() * t.element_size() for t in host_in.values())
-        d2h = sum(t.numel() * t.element_size() for t in host_out)
+        d2h = sum(t.numel() * t.element_size() for t in host_out[0])
+        copy_stream = torch.cuda.Stream()
+        copied = [torch.cuda.Event() for _ in sets]
+        used = [torch.cuda.Event() for _ in sets]
 
-        def e2e_step():
-            for k_, t in host_in.items():
-                getattr(wl, k_).copy_(t, non_blocking=True)
-            path.rescore(stream)
-            path.downstream(stream)
-            for hst, dv in zip(host_out, outs):
-                hst.copy_(dv, non_blocking=True)
+        def copy_in(i):
+            w_, _ = sets[i % 2]
+            with torch.cuda.stream(copy_stream):
+                if i >= 2:
+                    copy_stream.wait_event(used[i % 2])
+                for k_, t in host_in.items():
+                    getattr(w_, k_).copy_(t, non_blocking=True)
+                copied[i % 2].record(copy_stream)
 
-        for _ in range(2):
-            e2e_step()
+        def run_steps(n):
+            copy_in(0)
+            for i in range(n):
+                if i + 1 < n:
+                    copy_in(i + 1)
+                w_, p_ = sets[i % 2]
+                stream.wait_event(copied[i % 2])
+                p_.rescore(stream)
+                p_.downstream(stream)
+                used[i % 2].record(stream)
+                for hst, dv in zip(host_out[i % 2], (p_.bp, p_.ns, p_.bd, p_.mask)):
+                    hst.copy_(dv, non_blocking=True)
+
+        run_steps(2)
         torch.cuda.synchronize()
         barrier(world)
         e0 = torch.cuda.Event(enable_timing=True)
         e1 = torch.cuda.Event(enable_timing=True)
         e0.record(stream)
-        for _ in range(args.steps):
-            e2e_step()
+        copy_stream.wait_event(e0)
+        run_steps(args.steps)
         e1.record(stream)
         torch.cuda.synchronize()
         e2e_ms = max_over_ranks(e0.elapsed_time(e1), world)
+        ok = all(hdl.hdl_device_status(p_.ws, stream)[0] == hdl.HDL_OK for _, p_ in sets)
+        assert ok
+        assert torch.equal(host_out[0][0], host_out[1][0])   # both buffer sets agree
         e2e = {"value": world * N * args.steps / (e2e_ms / 1e3), "unit": "root tokens/s",
-               "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h}
+               "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+               "overlap": "inputs of step i+1 copied on a second stream during step i"}
+        del wl2, sets
 
     cpu = None
     if rank == 0 and not args.no_cpu:

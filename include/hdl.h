@@ -29,7 +29,7 @@
 extern "C" {
 #endif
 
-#define HDL_ABI_VERSION 1
+#define HDL_ABI_VERSION 2
 
 /* Exported symbols keep default visibility when the library is built with
  * -fvisibility=hidden. */
@@ -100,6 +100,43 @@ HDL_API hdl_status hdl_rescore(const void* h_orig, const void* h_hind,
                        int32_t vocab, float* logp_orig, float* logp_hind,
                        float* delta, void* workspace, size_t workspace_bytes,
                        void* cuda_stream);
+
+/* Options of hdl_rescore_ex.  A zero-initialised struct (or NULL) gives
+ * exactly hdl_rescore. */
+typedef struct {
+  /* [n_tokens] float outputs or NULL: the entropy (nats) of the next-token
+   * distribution, H_t = -sum_v p_t(v) log p_t(v), under the original / the
+   * hindsight context -- the ranking signal of the paper's Entropy selector
+   * (Section 4.1, "Rollout protocols"; the paper uses the original context).
+   * Computed in the same vocabulary walk (one more multiply-add per logit),
+   * as log Z - E_p[z]. */
+  float* entropy_orig;
+  float* entropy_hind;
+  /* Limit of each pipeline wait inside the kernel, ns; 0 = 4 s. */
+  uint64_t wait_timeout_ns;
+  /* Test hook, 0 in normal use.  Bit 0: the kernel's copy producer issues no
+   * loads, so the first pipeline wait runs out after wait_timeout_ns and the
+   * call reports HDL_ERR_TIMEOUT through hdl_device_status (nothing faults or
+   * hangs).  Other bits: HDL_ERR_INVALID_ARG. */
+  uint32_t fault_inject;
+  uint32_t reserved;
+} hdl_rescore_opts;
+
+/* Workspace of hdl_rescore_ex with these options (entropy outputs need
+ * 4 more bytes per row and vocabulary chunk); 0 for unsupported shapes. */
+HDL_API size_t hdl_rescore_ex_workspace_bytes(int64_t n_tokens, int32_t d, int32_t vocab,
+                                      hdl_dtype dt, const hdl_rescore_opts* opts);
+
+/* hdl_rescore with options (opts may be NULL).  Same arguments, layout,
+ * ownership and errors as hdl_rescore; the workspace must hold
+ * hdl_rescore_ex_workspace_bytes(..., opts) bytes. */
+HDL_API hdl_status hdl_rescore_ex(const void* h_orig, const void* h_hind,
+                          const void* w_lmhead, hdl_dtype dt,
+                          const int32_t* targets, int64_t n_tokens, int32_t d,
+                          int32_t vocab, float* logp_orig, float* logp_hind,
+                          float* delta, const hdl_rescore_opts* opts,
+                          void* workspace, size_t workspace_bytes,
+                          void* cuda_stream);
 
 /* Allocation-free variant of hdl_rescore (the paper has no counterpart: this
  * is an interface convenience).  It is for callers that must not allocate

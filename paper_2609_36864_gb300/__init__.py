@@ -21,7 +21,7 @@ __all__ = [
     "hdl_abi_version", "hdl_status_string", "hdl_rescore_workspace_bytes",
     "hdl_rescore", "hdl_device_status", "hdl_select_branches",
     "hdl_assign_continuations", "hdl_suffix_mask", "hdl_rescore_noalloc",
-    "HDL_STATIC_SCRATCH_BYTES",
+    "HDL_STATIC_SCRATCH_BYTES", "hdl_rescore_ex", "hdl_rescore_ex_workspace_bytes",
 ]
 
 HDL_OK, HDL_ERR_INVALID_ARG, HDL_ERR_UNSUPPORTED, HDL_ERR_WORKSPACE = 0, 1, 2, 3
@@ -44,6 +44,12 @@ class HdlError(RuntimeError):
         super().__init__(f"{fn} failed: {_status_name(code)} ({code})")
 
 
+class _RescoreOpts(ctypes.Structure):
+    _fields_ = [("entropy_orig", ctypes.c_void_p), ("entropy_hind", ctypes.c_void_p),
+                ("wait_timeout_ns", ctypes.c_uint64), ("fault_inject", ctypes.c_uint32),
+                ("reserved", ctypes.c_uint32)]
+
+
 class _SelectOpts(ctypes.Structure):
     _fields_ = [("min_gap", ctypes.c_int32), ("gap_mode", ctypes.c_int32),
                 ("lo", ctypes.c_int32), ("hi", ctypes.c_int32)]
@@ -60,6 +66,12 @@ def _declare(L):
     L.hdl_rescore.restype = ctypes.c_int
     L.hdl_rescore.argtypes = [vp, vp, vp, ctypes.c_int, vp, i64, i32, i32, vp, vp, vp,
                               vp, sz, vp]
+    L.hdl_rescore_ex_workspace_bytes.restype = sz
+    L.hdl_rescore_ex_workspace_bytes.argtypes = [i64, i32, i32, ctypes.c_int,
+                                                 ctypes.POINTER(_RescoreOpts)]
+    L.hdl_rescore_ex.restype = ctypes.c_int
+    L.hdl_rescore_ex.argtypes = [vp, vp, vp, ctypes.c_int, vp, i64, i32, i32, vp, vp, vp,
+                                 ctypes.POINTER(_RescoreOpts), vp, sz, vp]
     L.hdl_device_status.restype = ctypes.c_int
     L.hdl_device_status.argtypes = [vp, sz, vp, ctypes.POINTER(ctypes.c_uint32)]
     L.hdl_select_branches.restype = ctypes.c_int
@@ -186,6 +198,59 @@ def hdl_rescore(h_orig, h_hind, w_lmhead, targets, logp_orig=None, logp_hind=Non
                              _ptr(workspace), workspace.numel(), _stream(stream))
     _check("hdl_rescore", code)
     return logp_orig, logp_hind, delta, workspace
+
+
+def _opts(entropy_orig=None, entropy_hind=None, wait_timeout_ns=0, fault_inject=0):
+    return _RescoreOpts(None if entropy_orig is None else entropy_orig.data_ptr(),
+                        None if entropy_hind is None else entropy_hind.data_ptr(),
+                        int(wait_timeout_ns), int(fault_inject), 0)
+
+
+def hdl_rescore_ex_workspace_bytes(n_tokens: int, d: int, vocab: int, dtype=HDL_BF16,
+                                   entropy: bool = False) -> int:
+    if isinstance(dtype, torch.dtype):
+        dtype = HDL_BF16 if dtype == torch.bfloat16 else HDL_F32
+    o = _RescoreOpts(1 if entropy else None, None, 0, 0, 0)
+    return int(lib().hdl_rescore_ex_workspace_bytes(n_tokens, d, vocab, dtype, ctypes.byref(o)))
+
+
+def hdl_rescore_ex(h_orig, h_hind, w_lmhead, targets, logp_orig=None, logp_hind=None,
+                   delta=None, entropy_orig=None, entropy_hind=None, want_entropy=True,
+                   want_entropy_hind=False, wait_timeout_ns=0, fault_inject=0, workspace=None,
+                   stream=None):
+    """hdl_rescore plus the next-token entropies (Section 4.1, Entropy selector).
+
+    Returns (logp_orig, logp_hind, delta, entropy_orig, entropy_hind, workspace).
+    ``fault_inject`` is the library's test hook (see hdl_rescore_opts)."""
+    for t, n in ((h_orig, "h_orig"), (h_hind, "h_hind"), (w_lmhead, "w_lmhead")):
+        _dev(t, n)
+    _dev(targets, "targets", torch.int32)
+    dt = _hdl_dtype(h_orig)
+    N, d = h_orig.shape
+    V = w_lmhead.shape[0]
+    dev = h_orig.device
+
+    def out(t, want):
+        if t is None and want:
+            t = torch.empty(N, dtype=torch.float32, device=dev)
+        if t is not None:
+            _dev(t, "output", torch.float32)
+        return t
+    logp_orig, logp_hind = out(logp_orig, True), out(logp_hind, True)
+    delta = out(delta, True)
+    entropy_orig = out(entropy_orig, want_entropy)
+    entropy_hind = out(entropy_hind, want_entropy_hind)
+    o = _opts(entropy_orig, entropy_hind, wait_timeout_ns, fault_inject)
+    need = int(lib().hdl_rescore_ex_workspace_bytes(N, d, V, dt, ctypes.byref(o)))
+    if workspace is None:
+        workspace = torch.empty(max(need, 256), dtype=torch.uint8, device=dev)
+    _dev(workspace, "workspace", torch.uint8)
+    code = lib().hdl_rescore_ex(_ptr(h_orig), _ptr(h_hind), _ptr(w_lmhead), dt, _ptr(targets),
+                                N, d, V, _ptr(logp_orig), _ptr(logp_hind), _ptr(delta),
+                                ctypes.byref(o), _ptr(workspace), workspace.numel(),
+                                _stream(stream))
+    _check("hdl_rescore_ex", code)
+    return logp_orig, logp_hind, delta, entropy_orig, entropy_hind, workspace
 
 
 def hdl_device_status(workspace: torch.Tensor, stream=None):

@@ -30,6 +30,7 @@
 #include <cuda_runtime.h>
 #include <cudaTypedefs.h>
 
+#include <cfloat>
 #include <cmath>
 #include <cstdio>
 #include <cstdlib>
@@ -87,6 +88,7 @@ constexpr float kLn2 = 0.6931471805599453f;
 struct RescoreArgs {
   const int32_t* targets;
   float2* part;        // [num_chunks][2N] partial (max in log2 units, sum)
+  float* part_t;       // [num_chunks][2N] partial sum of p-weighted logits (entropy only)
   float* zt;           // [2N] target logit
   uint32_t* status;
   int64_t n_tokens;    // N rows per context
@@ -99,6 +101,7 @@ struct RescoreArgs {
   int32_t tiles_per_chunk;
   int32_t num_units;   // work units (per cluster in the cluster modes)
   int32_t group_m;     // M-tiles per rasterisation group (even)
+  uint32_t inject;     // test hook: bit 0 = the producer issues no copies
   uint64_t timeout_ns;
 };
 
@@ -156,7 +159,32 @@ __device__ __forceinline__ void lse_fold(const float (&x)[32], float& m2, float&
 // stage's empty barrier in both CTAs; mode 2: the even CTA's pair-MMA commit
 // arrives in both), and in mode 2 both CTAs' copies are counted on the even
 // CTA's full barrier and both epilogues release TMEM to the even CTA.
-template <bool kTf32, int M>
+// As lse_fold, also folding t = sum 2^(z log2e - m2) * z (the numerator of
+// E_p[z], for the entropy log Z - E_p[z]).
+__device__ __forceinline__ void lse_fold_ent(const float (&x)[32], float& m2, float& s,
+                                             float& t) {
+  float c[16];
+#pragma unroll
+  for (int j = 0; j < 16; ++j) c[j] = fmaxf(x[j], x[j + 16]);
+#pragma unroll
+  for (int w = 8; w >= 1; w >>= 1)
+#pragma unroll
+    for (int j = 0; j < w; ++j) c[j] = fmaxf(c[j], c[j + w]);
+  const float m_new = fmaxf(m2, c[0] * kLog2e);
+  float acc[4] = {0.f, 0.f, 0.f, 0.f}, acct[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+  for (int j = 0; j < 32; ++j) {
+    const float e = ex2_approx(fmaf(x[j], kLog2e, -m_new));
+    acc[j & 3] += e;
+    acct[j & 3] = fmaf(e, x[j], acct[j & 3]);
+  }
+  const float scale = ex2_approx(m2 - m_new);
+  s = fmaf(s, scale, (acc[0] + acc[1]) + (acc[2] + acc[3]));
+  t = fmaf(t, scale, (acct[0] + acct[1]) + (acct[2] + acct[3]));
+  m2 = m_new;
+}
+
+template <bool kTf32, int M, bool kEnt>
 __global__ void __launch_bounds__(kThreads, 1)
     rescore_lse_kernel(const __grid_constant__ CUtensorMap tm_h0,
                        const __grid_constant__ CUtensorMap tm_h1,
@@ -225,7 +253,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       int stage = 0;
       uint32_t phase = 0, pend = 0, pend_par = 0;
       bool ok = true;
-      for (int u = u_first; ok && u < a.num_units; u += u_step) {
+      const bool stall = (a.inject & 1u) != 0;   // test hook: issue nothing
+      for (int u = u_first; ok && !stall && u < a.num_units; u += u_step) {
         const Unit w = decode_unit<C::kCS>(u, a, rank);
         const CUtensorMap* tmA = w.ctx ? &tm_h1 : &tm_h0;
         for (int vt = w.vt0; ok && vt < w.vt1; ++vt) {
@@ -353,7 +382,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int64_t row = static_cast<int64_t>(w.row0) + r_in_tile;
       const bool in_range = row < a.n_tokens;
       const int32_t y = in_range ? __ldg(a.targets + row) : -1;
-      float m2 = -INFINITY, s = 0.f, zt = 0.f;
+      float m2 = -INFINITY, s = 0.f, zt = 0.f, tz = 0.f;
       bool found = false;
       for (int vt = w.vt0; vt < w.vt1; ++vt, ++tile) {
         const uint32_t buf = tile & 1u, use = (tile >> 1) & 1u;
@@ -374,10 +403,13 @@ __global__ void __launch_bounds__(kThreads, 1)
             tmem_load32(taddr + cc * 32, x);
             if (cc * 32 + 32 > ncols) {
 #pragma unroll
-              for (int j = 0; j < 32; ++j)
-                if (cc * 32 + j >= ncols) x[j] = -INFINITY;
+              for (int j = 0; j < 32; ++j)   // past the vocabulary: weight exactly 0
+                if (cc * 32 + j >= ncols) x[j] = -FLT_MAX;
             }
-            lse_fold(x, m2, s);
+            if constexpr (kEnt)
+              lse_fold_ent(x, m2, s, tz);
+            else
+              lse_fold(x, m2, s);
             const int rel = y - (v0 + cc * 32);
             if (static_cast<unsigned>(rel) < 32u) {
 #pragma unroll
@@ -400,6 +432,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int64_t rows_total = 2 * a.n_tokens;
         const int64_t g = w.ctx * a.n_tokens + row;
         a.part[static_cast<int64_t>(w.chunk) * rows_total + g] = make_float2(m2, s);
+        if constexpr (kEnt) a.part_t[static_cast<int64_t>(w.chunk) * rows_total + g] = tz;
         if (found) a.zt[g] = zt;
       }
     }
@@ -420,28 +453,33 @@ __global__ void __launch_bounds__(kThreads, 1)
 }
 
 // Merge the per-chunk partials of both contexts of token t and write
-// log p^0, log p^H and |Delta| (Eq. div).
+// log p^0, log p^H and |Delta| (Eq. div), and, when asked, the entropies
+// H = log Z - E_p[z] of both next-token distributions.
 __global__ void __launch_bounds__(256)
-    rescore_merge_kernel(const float2* __restrict__ part, const float* __restrict__ zt,
-                         const int32_t* __restrict__ targets, int64_t n, int32_t vocab,
-                         int32_t num_chunks, float* __restrict__ lp0,
+    rescore_merge_kernel(const float2* __restrict__ part, const float* __restrict__ part_t,
+                         const float* __restrict__ zt, const int32_t* __restrict__ targets,
+                         int64_t n, int32_t vocab, int32_t num_chunks, float* __restrict__ lp0,
                          float* __restrict__ lp1, float* __restrict__ delta,
-                         uint32_t* status) {
+                         float* __restrict__ ent0, float* __restrict__ ent1, uint32_t* status) {
   const int64_t rows_total = 2 * n;
   for (int64_t t = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; t < n;
        t += static_cast<int64_t>(gridDim.x) * blockDim.x) {
-    float lp[2];
+    float lp[2], ent[2];
 #pragma unroll
     for (int ctx = 0; ctx < 2; ++ctx) {
       const int64_t g = ctx * n + t;
       float M = -INFINITY;
       for (int c = 0; c < num_chunks; ++c) M = fmaxf(M, part[c * rows_total + g].x);
-      float S = 0.f;
+      float S = 0.f, T = 0.f;
       for (int c = 0; c < num_chunks; ++c) {
         const float2 p = part[c * rows_total + g];
-        S += p.y * exp2f(p.x - M);
+        const float sc = exp2f(p.x - M);
+        S += p.y * sc;
+        if (part_t) T += part_t[c * rows_total + g] * sc;
       }
-      lp[ctx] = zt[g] - (M + log2f(S)) * kLn2;
+      const float lse = (M + log2f(S)) * kLn2;
+      lp[ctx] = zt[g] - lse;
+      ent[ctx] = lse - T / S;
     }
     const int32_t y = targets[t];
     if (y < 0 || y >= vocab) {
@@ -451,6 +489,8 @@ __global__ void __launch_bounds__(256)
     lp0[t] = lp[0];
     lp1[t] = lp[1];
     if (delta) delta[t] = fabsf(lp[1] - lp[0]);
+    if (ent0) ent0[t] = ent[0];
+    if (ent1) ent1[t] = ent[1];
   }
 }
 
@@ -459,7 +499,7 @@ struct Geometry {
   int esize;
   int num_kb, num_m_ctx, num_m, num_vt, num_chunks, tiles_per_chunk;
   int64_t num_units;
-  size_t zt_off, part_off, total;
+  size_t zt_off, part_off, part_t_off, total, total_ent;
 };
 
 Geometry geometry(int64_t n, int32_t d, int32_t vocab, hdl_dtype dt) {
@@ -480,6 +520,8 @@ Geometry geometry(int64_t n, int32_t d, int32_t vocab, hdl_dtype dt) {
   g.zt_off = 256;
   g.part_off = g.zt_off + align_up(static_cast<size_t>(2 * n) * sizeof(float), 256);
   g.total = g.part_off + static_cast<size_t>(g.num_chunks) * static_cast<size_t>(2 * n) * sizeof(float2);
+  g.part_t_off = align_up(g.total, 256);
+  g.total_ent = g.part_t_off + static_cast<size_t>(g.num_chunks) * static_cast<size_t>(2 * n) * sizeof(float);
   return g;
 }
 
@@ -517,12 +559,12 @@ bool make_operand_map(CUtensorMap* m, const void* ptr, int64_t rows, int32_t d, 
 
 // One persistent CTA per SM (cluster modes: as many clusters of two as can
 // be resident at once).
-template <bool kTf32, int M>
+template <bool kTf32, int M, bool kEnt>
 hdl_status launch_rescore(const CUtensorMap& tm_h0, const CUtensorMap& tm_h1,
                           const CUtensorMap& tm_w, const RescoreArgs& a, int sms,
                           cudaStream_t st) {
   using C = Cfg<M>;
-  auto kern = rescore_lse_kernel<kTf32, M>;
+  auto kern = rescore_lse_kernel<kTf32, M, kEnt>;
   if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes) !=
       cudaSuccess)
     return HDL_ERR_CUDA;
@@ -590,25 +632,42 @@ extern "C" size_t hdl_rescore_workspace_bytes(int64_t n_tokens, int32_t d, int32
   return geometry(n_tokens, d, vocab, dt).total;
 }
 
-extern "C" hdl_status hdl_rescore(const void* h_orig, const void* h_hind, const void* w_lmhead,
-                                  hdl_dtype dt, const int32_t* targets, int64_t n_tokens,
-                                  int32_t d, int32_t vocab, float* logp_orig, float* logp_hind,
-                                  float* delta, void* workspace, size_t workspace_bytes,
-                                  void* cuda_stream) {
+extern "C" size_t hdl_rescore_ex_workspace_bytes(int64_t n_tokens, int32_t d, int32_t vocab,
+                                                 hdl_dtype dt, const hdl_rescore_opts* opts) {
+  if (check_shape(n_tokens, d, vocab, dt) != HDL_OK) return 0;
+  const Geometry g = geometry(n_tokens, d, vocab, dt);
+  const bool ent = opts && (opts->entropy_orig || opts->entropy_hind);
+  return ent ? g.total_ent : g.total;
+}
+
+extern "C" hdl_status hdl_rescore_ex(const void* h_orig, const void* h_hind,
+                                     const void* w_lmhead, hdl_dtype dt,
+                                     const int32_t* targets, int64_t n_tokens, int32_t d,
+                                     int32_t vocab, float* logp_orig, float* logp_hind,
+                                     float* delta, const hdl_rescore_opts* opts,
+                                     void* workspace, size_t workspace_bytes,
+                                     void* cuda_stream) {
   const hdl_status sh = check_shape(n_tokens, d, vocab, dt);
   if (sh != HDL_OK) return sh;
   if (n_tokens == 0) return HDL_OK;
+  hdl_rescore_opts o{};
+  if (opts) o = *opts;
+  if (o.fault_inject & ~1u) return HDL_ERR_INVALID_ARG;
+  const bool ent = o.entropy_orig || o.entropy_hind;
   if (!h_orig || !h_hind || !w_lmhead || !targets || !logp_orig || !logp_hind)
     return HDL_ERR_INVALID_ARG;
   if (!aligned_to(h_orig, 16) || !aligned_to(h_hind, 16) || !aligned_to(w_lmhead, 16) ||
       !aligned_to(targets, 4) || !aligned_to(logp_orig, 4) || !aligned_to(logp_hind, 4) ||
-      (delta && !aligned_to(delta, 4)))
+      (delta && !aligned_to(delta, 4)) || (o.entropy_orig && !aligned_to(o.entropy_orig, 4)) ||
+      (o.entropy_hind && !aligned_to(o.entropy_hind, 4)))
     return HDL_ERR_INVALID_ARG;
   const Geometry g = geometry(n_tokens, d, vocab, dt);
-  if (!workspace || !aligned_to(workspace, 256) || workspace_bytes < g.total)
+  if (!workspace || !aligned_to(workspace, 256) ||
+      workspace_bytes < (ent ? g.total_ent : g.total))
     return HDL_ERR_WORKSPACE;
 
-  const int mode = rescore_mode();
+  // the entropy variant always runs the default organisation
+  const int mode = ent ? kDefaultMode : rescore_mode();
   const int cs = mode == 0 ? 1 : 2;   // CTAs per cluster
   CUtensorMap tm_h0, tm_h1, tm_w;
   if (!make_operand_map(&tm_h0, h_orig, n_tokens, d, g.esize, kBM) ||
@@ -622,6 +681,7 @@ extern "C" hdl_status hdl_rescore(const void* h_orig, const void* h_hind, const 
   a.status = reinterpret_cast<uint32_t*>(ws);
   a.zt = reinterpret_cast<float*>(ws + g.zt_off);
   a.part = reinterpret_cast<float2*>(ws + g.part_off);
+  a.part_t = ent ? reinterpret_cast<float*>(ws + g.part_t_off) : nullptr;
   a.n_tokens = n_tokens;
   a.vocab = vocab;
   a.num_kb = g.num_kb;
@@ -632,7 +692,8 @@ extern "C" hdl_status hdl_rescore(const void* h_orig, const void* h_hind, const 
   a.tiles_per_chunk = g.tiles_per_chunk;
   a.num_units = static_cast<int32_t>(ceil_div(g.num_m, cs) * g.num_chunks);
   a.group_m = kGroupM;
-  a.timeout_ns = kDefaultTimeoutNs;
+  a.inject = o.fault_inject;
+  a.timeout_ns = o.wait_timeout_ns ? o.wait_timeout_ns : kDefaultTimeoutNs;
 
   cudaStream_t st = as_stream(cuda_stream);
   if (cudaMemsetAsync(a.status, 0, sizeof(uint32_t), st) != cudaSuccess) return HDL_ERR_CUDA;
@@ -641,24 +702,36 @@ extern "C" hdl_status hdl_rescore(const void* h_orig, const void* h_hind, const 
   if (sms <= 0) return HDL_ERR_CUDA;
   const bool tf32 = dt == HDL_F32;
   hdl_status ls;
-  if (mode == 0)
-    ls = tf32 ? launch_rescore<true, 0>(tm_h0, tm_h1, tm_w, a, sms, st)
-              : launch_rescore<false, 0>(tm_h0, tm_h1, tm_w, a, sms, st);
+  if (ent)
+    ls = tf32 ? launch_rescore<true, kDefaultMode, true>(tm_h0, tm_h1, tm_w, a, sms, st)
+              : launch_rescore<false, kDefaultMode, true>(tm_h0, tm_h1, tm_w, a, sms, st);
+  else if (mode == 0)
+    ls = tf32 ? launch_rescore<true, 0, false>(tm_h0, tm_h1, tm_w, a, sms, st)
+              : launch_rescore<false, 0, false>(tm_h0, tm_h1, tm_w, a, sms, st);
   else if (mode == 2)
-    ls = tf32 ? launch_rescore<true, 2>(tm_h0, tm_h1, tm_w, a, sms, st)
-              : launch_rescore<false, 2>(tm_h0, tm_h1, tm_w, a, sms, st);
+    ls = tf32 ? launch_rescore<true, 2, false>(tm_h0, tm_h1, tm_w, a, sms, st)
+              : launch_rescore<false, 2, false>(tm_h0, tm_h1, tm_w, a, sms, st);
   else
-    ls = tf32 ? launch_rescore<true, 1>(tm_h0, tm_h1, tm_w, a, sms, st)
-              : launch_rescore<false, 1>(tm_h0, tm_h1, tm_w, a, sms, st);
+    ls = tf32 ? launch_rescore<true, 1, false>(tm_h0, tm_h1, tm_w, a, sms, st)
+              : launch_rescore<false, 1, false>(tm_h0, tm_h1, tm_w, a, sms, st);
   if (ls != HDL_OK) return ls;
   if (launch_status() != HDL_OK) return HDL_ERR_CUDA;
 
   const int64_t mblocks = ceil_div(n_tokens, 256);
   const int mgrid = static_cast<int>(mblocks < 8 * sms ? mblocks : 8 * sms);
-  rescore_merge_kernel<<<mgrid, 256, 0, st>>>(a.part, a.zt, targets, n_tokens, vocab,
+  rescore_merge_kernel<<<mgrid, 256, 0, st>>>(a.part, a.part_t, a.zt, targets, n_tokens, vocab,
                                               g.num_chunks, logp_orig, logp_hind, delta,
-                                              a.status);
+                                              o.entropy_orig, o.entropy_hind, a.status);
   return launch_status();
+}
+
+extern "C" hdl_status hdl_rescore(const void* h_orig, const void* h_hind, const void* w_lmhead,
+                                  hdl_dtype dt, const int32_t* targets, int64_t n_tokens,
+                                  int32_t d, int32_t vocab, float* logp_orig, float* logp_hind,
+                                  float* delta, void* workspace, size_t workspace_bytes,
+                                  void* cuda_stream) {
+  return hdl_rescore_ex(h_orig, h_hind, w_lmhead, dt, targets, n_tokens, d, vocab, logp_orig,
+                        logp_hind, delta, nullptr, workspace, workspace_bytes, cuda_stream);
 }
 
 extern "C" hdl_status hdl_device_status(const void* workspace, size_t workspace_bytes,

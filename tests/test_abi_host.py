@@ -47,7 +47,7 @@ def test_only_declared_symbols_exported(L):
 
 def test_abi_version_and_names(L):
     import paper_2609_36864_gb300 as hdl
-    assert hdl.hdl_abi_version() == 1
+    assert hdl.hdl_abi_version() == 2
     assert hdl.hdl_status_string(0) == "HDL_OK"
     assert hdl.hdl_status_string(5) == "HDL_ERR_TIMEOUT"
     assert hdl.hdl_status_string(99) == "HDL_ERR_UNKNOWN"
@@ -153,3 +153,26 @@ def test_product_path_fails_loudly_without_library(monkeypatch, tmp_path):
     monkeypatch.setattr(hdl, "library_path", lambda: str(tmp_path / "missing.so"))
     with pytest.raises(RuntimeError, match="libhdl.so not found"):
         hdl.hdl_abi_version()
+
+
+def test_rescore_ex_options_and_workspace(L):
+    import paper_2609_36864_gb300 as hdl
+    n, d, V = 5000, 256, 9000
+    base = hdl.hdl_rescore_workspace_bytes(n, d, V)
+    assert hdl.hdl_rescore_ex_workspace_bytes(n, d, V) == base
+    ent = hdl.hdl_rescore_ex_workspace_bytes(n, d, V, entropy=True)
+    cdiv = lambda a, b: -(-a // b)
+    num_m, nvt, tpc = 2 * cdiv(n, 128), cdiv(V, 256), 16
+    while tpc > 1 and num_m * cdiv(nvt, tpc) < 1216:
+        tpc //= 2
+    assert ent == cdiv(base, 256) * 256 + cdiv(nvt, tpc) * 2 * n * 4
+    o = hdl._RescoreOpts(None, None, 0, 2, 0)          # unknown fault bit
+    assert L.hdl_rescore_ex(P, P, P, 0, P, 16, 64, 100, P, P, None, ctypes.byref(o), P,
+                            1 << 40, None) == 1
+    o = hdl._RescoreOpts(0x10002, None, 0, 0, 0)       # misaligned entropy output
+    assert L.hdl_rescore_ex(P, P, P, 0, P, 16, 64, 100, P, P, None, ctypes.byref(o), P,
+                            1 << 40, None) == 1
+    o = hdl._RescoreOpts(0x10000, None, 0, 0, 0)       # entropy needs the larger workspace
+    small = hdl.hdl_rescore_workspace_bytes(16, 64, 100)
+    assert L.hdl_rescore_ex(P, P, P, 0, P, 16, 64, 100, P, P, None, ctypes.byref(o), P,
+                            small, None) == 3

@@ -153,3 +153,27 @@ def test_rescore_cta_modes_agree_bitwise(hdl, tmp_path):
     y = wl.targets.cpu().numpy()
     assert_logp_close(outs["0"][0][0], oracle_logprobs(to_f64(wl.h_orig), W, y), "modes orig")
     assert_logp_close(outs["0"][0][1], oracle_logprobs(to_f64(wl.h_hind), W, y), "modes hind")
+
+
+@pytest.mark.parametrize("n,d,V,dt", [(300, 256, 4097, "bf16"), (129, 128, 257, "bf16"),
+                                      (1000, 1024, 8192, "bf16"), (200, 256, 5000, "f32"),
+                                      (1, 64, 1, "bf16")])
+def test_rescore_entropy(hdl, n, d, V, dt):
+    """Next-token entropies of both contexts (the Entropy selector's signal,
+    Section 4.1) against the oracle; asking for them leaves the log-probs
+    unchanged bit for bit."""
+    spec = hdl_synth.small_spec(f"e{n}_{d}_{V}", n_roots=1, t_lo=n, t_hi=n, d=d, vocab=V,
+                                dtype=dt, seed=7 * n + V)
+    wl = hdl_synth.generate(spec, device="cuda")
+    lp0, lp1, de, e0, e1, ws = hdl.hdl_rescore_ex(wl.h_orig, wl.h_hind, wl.w, wl.targets,
+                                                  want_entropy_hind=True)
+    assert hdl.hdl_device_status(ws)[0] == hdl.HDL_OK
+    r = hdl.hdl_rescore(wl.h_orig, wl.h_hind, wl.w, wl.targets)
+    assert torch.equal(lp0, r[0]) and torch.equal(lp1, r[1]) and torch.equal(de, r[2])
+    import oracle
+    W = to_f64(wl.w)
+    h0, h1 = to_f64(wl.h_orig), to_f64(wl.h_hind)
+    assert_logp_close(e0.cpu().numpy(), oracle.next_token_entropy(h0, W), "entropy orig")
+    assert_logp_close(e1.cpu().numpy(), oracle.next_token_entropy(h1, W), "entropy hind")
+    if V == 1:
+        assert torch.all(e0.abs() < 1e-6)

@@ -101,3 +101,20 @@ def test_workload_sampled(hdl, which):
     # properties that hold at any size
     assert np.all(out["lp0"] <= 1e-5) and np.all(out["lp1"] <= 1e-5)
     assert np.all(np.isfinite(out["delta"])) and np.all(out["delta"] >= 0)
+
+
+@pytest.mark.parametrize("name", ["tiny", "math"])
+def test_workload_entropy_selector(hdl, name):
+    """The Entropy selector of Section 4.1: rank positions by the entropy of
+    the next-token distribution under the original context, through the same
+    selection kernel; branch sets match the oracle's within the band."""
+    wl = hdl_synth.generate(hdl_synth.SPECS[name], device="cuda")
+    lp0, lp1, de, e0, _, ws = hdl.hdl_rescore_ex(wl.h_orig, wl.h_hind, wl.w, wl.targets)
+    bp, ns, bd = hdl.hdl_select_branches(e0, wl.valid, wl.root_offsets, wl.spec.k)
+    assert hdl.hdl_device_status(ws)[0] == hdl.HDL_OK
+    ref = oracle.next_token_entropy(to_f64(wl.h_orig), to_f64(wl.w)) if name == "tiny" else \
+        np.concatenate([oracle.next_token_entropy(to_f64(wl.h_orig[s:s + 2048]), to_f64(wl.w))
+                        for s in range(0, wl.n_tokens, 2048)])
+    assert_logp_close(e0.cpu().numpy(), ref, name + " entropy")
+    check_selection_band(bp.cpu().numpy(), ns.cpu().numpy(), ref, wl.valid.cpu().numpy(),
+                         wl.root_offsets.cpu().numpy(), wl.spec.k)
