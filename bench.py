@@ -199,6 +199,13 @@ def max_over_ranks(x: float, world: int) -> float:
     return float(t.item())
 
 
+def aggregate_value(world: int, n_tokens_per_rank: int, steps: int, max_ms: float) -> float:
+    """Whole-job root tokens/s: every rank re-scores its own workload of
+    n_tokens_per_rank tokens per step (weak scaling); the slowest rank's
+    time counts."""
+    return world * n_tokens_per_rank * steps / (max_ms / 1e3)
+
+
 def cpu_oracle_sample(wl, seconds: float, rng_seed: int = 0):
     """Time the fp64 oracle on sampled tokens of the workload: log-probs of
     both contexts for a growing sample until ``seconds`` of CPU work, plus
@@ -321,7 +328,7 @@ def run_gpu(args, world, rank, local):
     assert code == hdl.HDL_OK, (code, raw)
     total_ms = max_over_ranks(t_start.elapsed_time(t_end), world)
     rescore_ms = float(np.mean([a.elapsed_time(b_) for a, b_ in ev]))
-    value = world * N * args.steps / (total_ms / 1e3)
+    value = aggregate_value(world, N, args.steps, total_ms)
 
     # ---- end to end: every step's inputs are copied host -> device from
     # pinned memory and its results device -> host.  Inputs are double
@@ -379,7 +386,7 @@ def run_gpu(args, world, rank, local):
         ok = all(hdl.hdl_device_status(p_.ws, stream)[0] == hdl.HDL_OK for _, p_ in sets)
         assert ok
         assert torch.equal(host_out[0][0], host_out[1][0])   # both buffer sets agree
-        e2e = {"value": world * N * args.steps / (e2e_ms / 1e3), "unit": "root tokens/s",
+        e2e = {"value": aggregate_value(world, N, args.steps, e2e_ms), "unit": "root tokens/s",
                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                "overlap": "inputs of step i+1 copied on a second stream during step i"}
         del wl2, sets

@@ -138,6 +138,83 @@ HDL_API hdl_status hdl_rescore_ex(const void* h_orig, const void* h_hind,
                           void* workspace, size_t workspace_bytes,
                           void* cuda_stream);
 
+/* ------------------------------------------------------------------------
+ * Vocabulary-parallel re-scoring (a tensor-parallel LM head: each GPU holds
+ * rows [vocab_offset, vocab_offset + vocab_shard) of W).  The softmax
+ * normaliser of Section 3.1 splits over shards exactly: with per-shard
+ * m_p = max z (log2 units) and s_p = sum 2^(z log2e - m_p),
+ *   log Z = ln2 * (M + log2 sum_p s_p 2^(m_p - M)),  M = max_p m_p,
+ * so one exchange of 16 bytes per row and context (e.g. an all-gather)
+ * followed by hdl_merge_vocab_shards gives the same log-probs as one GPU.
+ *
+ * hdl_rescore_shard writes stats, [2][n_tokens] float4 (context 0 = original,
+ * 16-byte aligned): x = m_p, y = s_p, z = the target logit z_{y_t} if this
+ * shard holds y_t else NaN, w = sum 2^(z log2e - m_p) * z (for the entropy).
+ * Arguments otherwise as hdl_rescore (w_shard is [vocab_shard, d]; targets
+ * are global ids); the workspace holds
+ * hdl_rescore_shard_workspace_bytes(n_tokens, d, vocab_shard, dt) bytes. */
+HDL_API size_t hdl_rescore_shard_workspace_bytes(int64_t n_tokens, int32_t d,
+                                         int32_t vocab_shard, hdl_dtype dt);
+
+HDL_API hdl_status hdl_rescore_shard(const void* h_orig, const void* h_hind,
+                             const void* w_shard, hdl_dtype dt,
+                             const int32_t* targets, int64_t n_tokens, int32_t d,
+                             int32_t vocab_shard, int32_t vocab_offset,
+                             float* stats, void* workspace,
+                             size_t workspace_bytes, void* cuda_stream);
+
+/* Merge n_shards shards' stats, laid out back to back (shard p at
+ * stats + p * 2 * n_tokens * 4 floats), into log-probs, |Delta| and
+ * (optional, NULL to skip) entropies.  A token whose target no shard holds
+ * gets NaN log-probs.  delta, entropy_orig, entropy_hind may be NULL. */
+HDL_API hdl_status hdl_merge_vocab_shards(const float* stats, int32_t n_shards,
+                                  int64_t n_tokens, float* logp_orig,
+                                  float* logp_hind, float* delta,
+                                  float* entropy_orig, float* entropy_hind,
+                                  void* cuda_stream);
+
+/* ------------------------------------------------------------------------
+ * The update after branch selection: group-relative advantages and the
+ * clipped, token-aggregated policy loss on the suffix-only masks.
+ *
+ * Section 3: A_j = R_j - (1/G) sum_{k in group} R_k (no standard-deviation
+ * normalisation, Section 4.1); the group's roots and continuations form one
+ * group (Section 3.3).  Section 4.1 "Training": asymmetric clipping with
+ * thresholds 0.2 / 0.28, no KL penalty, losses aggregated at the token level:
+ *   r_t = exp(logp_new_t - logp_old_t),
+ *   obj_t = min(r_t A_j, clip(r_t, 1 - eps_low, 1 + eps_high) A_j),
+ *   loss = - sum_t mask_t obj_t / sum_t mask_t,
+ *   grad_t = d loss / d logp_new_t (= -mask_t r_t A_j / sum mask when the
+ *            unclipped term is the minimum, else 0).
+ *
+ *   logp_new, logp_old  [n_tokens] float, packed trajectories.
+ *   mask            [n_tokens] uint8: the loss mask (hdl_suffix_mask for
+ *                   continuations, the valid mask for roots).
+ *   traj_offsets    [n_traj + 1] int64: trajectory j = tokens
+ *                   [traj_offsets[j], traj_offsets[j+1]); they should cover
+ *                   [0, n_tokens) (tokens outside every trajectory carry no loss).
+ *   rewards         [n_traj] float verifier rewards.
+ *   group_offsets   [n_groups + 1] int32: group g = trajectories
+ *                   [group_offsets[g], group_offsets[g+1]).
+ *   eps_low, eps_high  clip thresholds, 0 <= eps_low < 1, eps_high >= 0.
+ *   advantages      [n_traj] float out (trajectories outside every group are
+ *                   not written).
+ *   grad            [n_tokens] float out or NULL.
+ *   stats           [4] float out: loss, masked tokens, fraction of masked
+ *                   tokens whose clipped term is strictly smaller, mean ratio.
+ *   workspace       hdl_grpo_loss_workspace_bytes() bytes, 256-byte aligned.
+ * The loss is reduced in double precision in a fixed order. */
+HDL_API size_t hdl_grpo_loss_workspace_bytes(void);
+
+HDL_API hdl_status hdl_grpo_loss(const float* logp_new, const float* logp_old,
+                         const uint8_t* mask, int64_t n_tokens,
+                         const int64_t* traj_offsets, int32_t n_traj,
+                         const float* rewards, const int32_t* group_offsets,
+                         int32_t n_groups, float eps_low, float eps_high,
+                         float* advantages, float* grad, float* stats,
+                         void* workspace, size_t workspace_bytes,
+                         void* cuda_stream);
+
 /* Allocation-free variant of hdl_rescore (the paper has no counterpart: this
  * is an interface convenience).  It is for callers that must not allocate
  * device memory while they run: plugin "enqueue" callbacks of inference

@@ -27,6 +27,11 @@ Functions and the passages they follow (arXiv 2609.36864):
   suffix_mask            Section 3.3: a root's loss covers its generated
                          tokens; a continuation's loss covers only the newly
                          sampled tokens y~_{>= i} of Eq. (branch-sampling).
+  group_advantages       Section 3: A_j = R_j - mean of the group's rewards (no
+                         standard-deviation normalisation, Section 4.1).
+  grpo_token_loss        Section 4.1 "Training": the clipped policy objective
+                         with asymmetric clipping (0.2 / 0.28), no KL term,
+                         aggregated over tokens, on the suffix-only masks.
 
 Readings where the paper is silent (each is also listed in the design notes):
   * ties in s_i go to the lower position;
@@ -55,7 +60,8 @@ import numpy as np
 __all__ = [
     "widen", "target_logprobs", "hindsight_divergence", "next_token_entropy",
     "select_branches",
-    "allocate_counts", "assign_continuations", "suffix_mask",
+    "allocate_counts", "assign_continuations", "suffix_mask", "group_advantages",
+    "grpo_token_loss",
 ]
 
 
@@ -227,3 +233,61 @@ def suffix_mask(cont_branch, cont_offsets, cont_valid=None) -> np.ndarray:
             m &= np.asarray(cont_valid[start:end]) != 0
         mask[start:end] = m
     return mask
+
+
+def group_advantages(rewards, group_offsets) -> np.ndarray:
+    """A_j = R_j - (1/G) sum_{k in group} R_k for every trajectory (Section 3).
+
+    Group g holds trajectories [group_offsets[g], group_offsets[g+1]) -- its
+    roots and their continuations (Section 3.3: they form one group).
+    """
+    R = np.asarray(rewards, dtype=np.float64)
+    offs = np.asarray(group_offsets, dtype=np.int64)
+    A = np.zeros(len(R))
+    for g in range(len(offs) - 1):
+        lo, hi = int(offs[g]), int(offs[g + 1])
+        if hi > lo:
+            A[lo:hi] = R[lo:hi] - R[lo:hi].mean()
+    return A
+
+
+def grpo_token_loss(logp_new, logp_old, mask, traj_offsets, advantages,
+                    eps_low: float = 0.2, eps_high: float = 0.28, decide_in=np.float64):
+    """Clipped policy loss aggregated over tokens (Section 4.1).
+
+    For token t of trajectory j with mask m_t (Section 3.3's suffix-only mask):
+      r_t   = exp(logp_new_t - logp_old_t)
+      obj_t = min(r_t A_j, clip(r_t, 1 - eps_low, 1 + eps_high) A_j)
+      loss  = - sum_t m_t obj_t / sum_t m_t
+    and grad_t = d loss / d logp_new_t, which is -m_t r_t A_j / sum m when the
+    unclipped term is the minimum (ties included) and 0 otherwise.
+    Returns (loss, grad, stats) with stats = (masked tokens, fraction of masked
+    tokens whose clipped term is strictly the minimum, mean masked ratio).
+    ``decide_in`` is the precision in which "which term is the minimum" is
+    decided (the values themselves stay float64): a GPU comparison passes
+    np.float32, the precision the kernel decides in.
+    """
+    lpn = np.asarray(logp_new, dtype=np.float64)
+    lpo = np.asarray(logp_old, dtype=np.float64)
+    m = np.asarray(mask) != 0
+    offs = np.asarray(traj_offsets, dtype=np.int64)
+    A = np.zeros(len(lpn))
+    for j in range(len(offs) - 1):
+        A[int(offs[j]):int(offs[j + 1])] = advantages[j]
+    r = np.exp(lpn - lpo)
+    unclipped = r * A
+    clipped = np.clip(r, 1.0 - eps_low, 1.0 + eps_high) * A
+    obj = np.minimum(unclipped, clipped)
+    n = int(m.sum())
+    if n == 0:
+        return 0.0, np.zeros(len(lpn)), (0, 0.0, 0.0)
+    loss = -obj[m].sum() / n
+    r_d = np.exp(lpn.astype(decide_in) - lpo.astype(decide_in))
+    A_d = A.astype(decide_in)
+    lo_d, hi_d = decide_in(1.0) - decide_in(eps_low), decide_in(1.0) + decide_in(eps_high)
+    active = (r_d * A_d) <= (np.clip(r_d, lo_d, hi_d) * A_d)
+    obj = np.where(active, unclipped, clipped)
+    loss = -obj[m].sum() / n
+    grad = np.where(m & active, -r * A / n, 0.0)
+    clip_frac = float((~active[m]).sum()) / n
+    return float(loss), grad, (n, clip_frac, float(r[m].mean()))

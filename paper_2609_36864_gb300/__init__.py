@@ -22,6 +22,8 @@ __all__ = [
     "hdl_rescore", "hdl_device_status", "hdl_select_branches",
     "hdl_assign_continuations", "hdl_suffix_mask", "hdl_rescore_noalloc",
     "HDL_STATIC_SCRATCH_BYTES", "hdl_rescore_ex", "hdl_rescore_ex_workspace_bytes",
+    "hdl_rescore_shard", "hdl_rescore_shard_workspace_bytes", "hdl_merge_vocab_shards",
+    "hdl_grpo_loss", "hdl_grpo_loss_workspace_bytes",
 ]
 
 HDL_OK, HDL_ERR_INVALID_ARG, HDL_ERR_UNSUPPORTED, HDL_ERR_WORKSPACE = 0, 1, 2, 3
@@ -72,6 +74,18 @@ def _declare(L):
     L.hdl_rescore_ex.restype = ctypes.c_int
     L.hdl_rescore_ex.argtypes = [vp, vp, vp, ctypes.c_int, vp, i64, i32, i32, vp, vp, vp,
                                  ctypes.POINTER(_RescoreOpts), vp, sz, vp]
+    L.hdl_rescore_shard_workspace_bytes.restype = sz
+    L.hdl_rescore_shard_workspace_bytes.argtypes = [i64, i32, i32, ctypes.c_int]
+    L.hdl_rescore_shard.restype = ctypes.c_int
+    L.hdl_rescore_shard.argtypes = [vp, vp, vp, ctypes.c_int, vp, i64, i32, i32, i32, vp, vp,
+                                    sz, vp]
+    L.hdl_merge_vocab_shards.restype = ctypes.c_int
+    L.hdl_merge_vocab_shards.argtypes = [vp, i32, i64, vp, vp, vp, vp, vp, vp]
+    L.hdl_grpo_loss_workspace_bytes.restype = sz
+    L.hdl_grpo_loss_workspace_bytes.argtypes = []
+    L.hdl_grpo_loss.restype = ctypes.c_int
+    L.hdl_grpo_loss.argtypes = [vp, vp, vp, i64, vp, i32, vp, vp, i32, ctypes.c_float,
+                                ctypes.c_float, vp, vp, vp, vp, sz, vp]
     L.hdl_device_status.restype = ctypes.c_int
     L.hdl_device_status.argtypes = [vp, sz, vp, ctypes.POINTER(ctypes.c_uint32)]
     L.hdl_select_branches.restype = ctypes.c_int
@@ -352,3 +366,93 @@ def hdl_rescore_noalloc(h_orig, h_hind, w_lmhead, targets, logp_orig, logp_hind,
                                      _ptr(delta), ctypes.byref(scratch), _stream(stream))
     _check("hdl_rescore_noalloc", code)
     return scratch.value
+
+
+def hdl_rescore_shard_workspace_bytes(n_tokens: int, d: int, vocab_shard: int,
+                                      dtype=HDL_BF16) -> int:
+    if isinstance(dtype, torch.dtype):
+        dtype = HDL_BF16 if dtype == torch.bfloat16 else HDL_F32
+    return int(lib().hdl_rescore_shard_workspace_bytes(n_tokens, d, vocab_shard, dtype))
+
+
+def hdl_rescore_shard(h_orig, h_hind, w_shard, targets, vocab_offset: int, stats=None,
+                      workspace=None, stream=None):
+    """Per-row statistics of one vocabulary shard of the LM head: a
+    [2, n_tokens, 4] float tensor (max in log2 units, sum, target logit or NaN,
+    entropy numerator), to be exchanged and merged by hdl_merge_vocab_shards."""
+    for t, n in ((h_orig, "h_orig"), (h_hind, "h_hind"), (w_shard, "w_shard")):
+        _dev(t, n)
+    _dev(targets, "targets", torch.int32)
+    dt = _hdl_dtype(h_orig)
+    N, d = h_orig.shape
+    Vs = w_shard.shape[0]
+    if stats is None:
+        stats = torch.empty((2, N, 4), dtype=torch.float32, device=h_orig.device)
+    _dev(stats, "stats", torch.float32)
+    need = hdl_rescore_shard_workspace_bytes(N, d, Vs, dt)
+    if workspace is None:
+        workspace = torch.empty(max(need, 256), dtype=torch.uint8, device=h_orig.device)
+    code = lib().hdl_rescore_shard(_ptr(h_orig), _ptr(h_hind), _ptr(w_shard), dt, _ptr(targets),
+                                   N, d, Vs, int(vocab_offset), _ptr(stats), _ptr(workspace),
+                                   workspace.numel(), _stream(stream))
+    _check("hdl_rescore_shard", code)
+    return stats, workspace
+
+
+def hdl_merge_vocab_shards(stats, logp_orig=None, logp_hind=None, delta=None,
+                           entropy_orig=None, entropy_hind=None, want_entropy=True,
+                           stream=None):
+    """Merge stacked shard statistics [P, 2, n_tokens, 4] into log-probs,
+    |Delta| and entropies: returns (logp_orig, logp_hind, delta, H_orig, H_hind)."""
+    _dev(stats, "stats", torch.float32)
+    P, two, N, four = stats.shape
+    if two != 2 or four != 4:
+        raise ValueError("stats must be [n_shards, 2, n_tokens, 4]")
+    dev = stats.device
+
+    def out(t, want=True):
+        if t is None and want:
+            t = torch.empty(N, dtype=torch.float32, device=dev)
+        return t
+    logp_orig, logp_hind, delta = out(logp_orig), out(logp_hind), out(delta)
+    entropy_orig, entropy_hind = out(entropy_orig, want_entropy), out(entropy_hind, want_entropy)
+    code = lib().hdl_merge_vocab_shards(_ptr(stats), P, N, _ptr(logp_orig), _ptr(logp_hind),
+                                        _ptr(delta), _ptr(entropy_orig), _ptr(entropy_hind),
+                                        _stream(stream))
+    _check("hdl_merge_vocab_shards", code)
+    return logp_orig, logp_hind, delta, entropy_orig, entropy_hind
+
+
+def hdl_grpo_loss_workspace_bytes() -> int:
+    return int(lib().hdl_grpo_loss_workspace_bytes())
+
+
+def hdl_grpo_loss(logp_new, logp_old, mask, traj_offsets, rewards, group_offsets,
+                  eps_low: float = 0.2, eps_high: float = 0.28, advantages=None, grad=None,
+                  want_grad=True, stats=None, workspace=None, stream=None):
+    """Group advantages and the clipped token-level policy loss (Section 4.1).
+
+    Returns (advantages [J], grad [T] or None, stats [4] = loss, masked
+    tokens, clipped fraction, mean ratio), all on the device."""
+    _dev(logp_new, "logp_new", torch.float32)
+    _dev(logp_old, "logp_old", torch.float32)
+    _dev(mask, "mask", torch.uint8)
+    _dev(traj_offsets, "traj_offsets", torch.int64)
+    _dev(rewards, "rewards", torch.float32)
+    _dev(group_offsets, "group_offsets", torch.int32)
+    dev = logp_new.device
+    T, J, G = logp_new.numel(), traj_offsets.numel() - 1, group_offsets.numel() - 1
+    if advantages is None:
+        advantages = torch.zeros(J, dtype=torch.float32, device=dev)
+    if grad is None and want_grad:
+        grad = torch.empty(T, dtype=torch.float32, device=dev)
+    if stats is None:
+        stats = torch.empty(4, dtype=torch.float32, device=dev)
+    if workspace is None:
+        workspace = torch.empty(hdl_grpo_loss_workspace_bytes(), dtype=torch.uint8, device=dev)
+    code = lib().hdl_grpo_loss(_ptr(logp_new), _ptr(logp_old), _ptr(mask), T, _ptr(traj_offsets),
+                               J, _ptr(rewards), _ptr(group_offsets), G, float(eps_low),
+                               float(eps_high), _ptr(advantages), _ptr(grad), _ptr(stats),
+                               _ptr(workspace), workspace.numel(), _stream(stream))
+    _check("hdl_grpo_loss", code)
+    return advantages, grad, stats

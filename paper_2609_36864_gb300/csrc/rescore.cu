@@ -101,6 +101,7 @@ struct RescoreArgs {
   int32_t tiles_per_chunk;
   int32_t num_units;   // work units (per cluster in the cluster modes)
   int32_t group_m;     // M-tiles per rasterisation group (even)
+  int32_t target_offset;  // targets are shifted by this (vocabulary shards)
   uint32_t inject;     // test hook: bit 0 = the producer issues no copies
   uint64_t timeout_ns;
 };
@@ -381,7 +382,11 @@ __global__ void __launch_bounds__(kThreads, 1)
       const Unit w = decode_unit<C::kCS>(u, a, rank);
       const int64_t row = static_cast<int64_t>(w.row0) + r_in_tile;
       const bool in_range = row < a.n_tokens;
-      const int32_t y = in_range ? __ldg(a.targets + row) : -1;
+      // the target column relative to this call's vocabulary; one outside it
+      // (another shard's, or a bad id) is never gathered, not even from the
+      // masked tail of the last tile
+      int32_t y = in_range ? __ldg(a.targets + row) - a.target_offset : -1;
+      if (y < 0 || y >= a.vocab) y = -1;
       float m2 = -INFINITY, s = 0.f, zt = 0.f, tz = 0.f;
       bool found = false;
       for (int vt = w.vt0; vt < w.vt1; ++vt, ++tile) {
@@ -485,6 +490,63 @@ __global__ void __launch_bounds__(256)
     if (y < 0 || y >= vocab) {
       lp[0] = lp[1] = __int_as_float(0x7fc00000);
       atomicOr(status, kStatusBadTarget);
+    }
+    lp0[t] = lp[0];
+    lp1[t] = lp[1];
+    if (delta) delta[t] = fabsf(lp[1] - lp[0]);
+    if (ent0) ent0[t] = ent[0];
+    if (ent1) ent1[t] = ent[1];
+  }
+}
+
+// Per-row statistics of one vocabulary shard: the chunk partials folded to
+// (m, s, zt, t): max in log2 units, sum of 2^(z log2e - m), the target logit
+// (NaN when the target is outside this shard) and sum of 2^(z log2e - m) z.
+__global__ void __launch_bounds__(256)
+    shard_stats_kernel(const float2* __restrict__ part, const float* __restrict__ part_t,
+                       const float* __restrict__ zt, int64_t n, int32_t num_chunks,
+                       float4* __restrict__ stats) {
+  const int64_t rows_total = 2 * n;
+  for (int64_t g = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; g < rows_total;
+       g += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+    float M = -INFINITY;
+    for (int c = 0; c < num_chunks; ++c) M = fmaxf(M, part[c * rows_total + g].x);
+    float S = 0.f, T = 0.f;
+    for (int c = 0; c < num_chunks; ++c) {
+      const float sc = exp2f(part[c * rows_total + g].x - M);
+      S += part[c * rows_total + g].y * sc;
+      T += part_t[c * rows_total + g] * sc;
+    }
+    stats[g] = make_float4(M, S, zt[g], T);
+  }
+}
+
+// Merge the statistics of n_shards vocabulary shards (stats[p][ctx][t]).
+__global__ void __launch_bounds__(256)
+    merge_shards_kernel(const float4* __restrict__ stats, int32_t n_shards, int64_t n,
+                        float* __restrict__ lp0, float* __restrict__ lp1,
+                        float* __restrict__ delta, float* __restrict__ ent0,
+                        float* __restrict__ ent1) {
+  const int64_t rows_total = 2 * n;
+  for (int64_t t = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; t < n;
+       t += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+    float lp[2], ent[2];
+#pragma unroll
+    for (int ctx = 0; ctx < 2; ++ctx) {
+      const int64_t g = ctx * n + t;
+      float M = -INFINITY;
+      for (int p = 0; p < n_shards; ++p) M = fmaxf(M, stats[p * rows_total + g].x);
+      float S = 0.f, T = 0.f, z = __int_as_float(0x7fc00000);
+      for (int p = 0; p < n_shards; ++p) {
+        const float4 q = stats[p * rows_total + g];
+        const float sc = exp2f(q.x - M);
+        S += q.y * sc;
+        T += q.w * sc;
+        if (!isnan(q.z) && isnan(z)) z = q.z;
+      }
+      const float lse = (M + log2f(S)) * kLn2;
+      lp[ctx] = z - lse;
+      ent[ctx] = lse - T / S;
     }
     lp0[t] = lp[0];
     lp1[t] = lp[1];
@@ -791,4 +853,96 @@ extern "C" hdl_status hdl_rescore_noalloc(const void* h_orig, const void* h_hind
   if (scratch_out) *scratch_out = ws;
   return hdl_rescore(h_orig, h_hind, w_lmhead, dt, targets, n_tokens, d, vocab, logp_orig,
                      logp_hind, delta, ws, HDL_STATIC_SCRATCH_BYTES, cuda_stream);
+}
+
+// ---------------------------------------------------------------------------
+// Vocabulary-parallel re-scoring: one shard of W per call, statistics out.
+extern "C" size_t hdl_rescore_shard_workspace_bytes(int64_t n_tokens, int32_t d,
+                                                    int32_t vocab_shard, hdl_dtype dt) {
+  if (check_shape(n_tokens, d, vocab_shard, dt) != HDL_OK) return 0;
+  return geometry(n_tokens, d, vocab_shard, dt).total_ent;
+}
+
+extern "C" hdl_status hdl_rescore_shard(const void* h_orig, const void* h_hind,
+                                        const void* w_shard, hdl_dtype dt,
+                                        const int32_t* targets, int64_t n_tokens, int32_t d,
+                                        int32_t vocab_shard, int32_t vocab_offset, float* stats,
+                                        void* workspace, size_t workspace_bytes,
+                                        void* cuda_stream) {
+  const hdl_status sh = check_shape(n_tokens, d, vocab_shard, dt);
+  if (sh != HDL_OK) return sh;
+  if (vocab_offset < 0) return HDL_ERR_INVALID_ARG;
+  if (n_tokens == 0) return HDL_OK;
+  if (!h_orig || !h_hind || !w_shard || !targets || !stats) return HDL_ERR_INVALID_ARG;
+  if (!aligned_to(h_orig, 16) || !aligned_to(h_hind, 16) || !aligned_to(w_shard, 16) ||
+      !aligned_to(targets, 4) || !aligned_to(stats, 16))
+    return HDL_ERR_INVALID_ARG;
+  const Geometry g = geometry(n_tokens, d, vocab_shard, dt);
+  if (!workspace || !aligned_to(workspace, 256) || workspace_bytes < g.total_ent)
+    return HDL_ERR_WORKSPACE;
+  constexpr int cs = Cfg<kDefaultMode>::kCS;
+  CUtensorMap tm_h0, tm_h1, tm_w;
+  if (!make_operand_map(&tm_h0, h_orig, n_tokens, d, g.esize, kBM) ||
+      !make_operand_map(&tm_h1, h_hind, n_tokens, d, g.esize, kBM) ||
+      !make_operand_map(&tm_w, w_shard, vocab_shard, d, g.esize, kBN / cs))
+    return HDL_ERR_CUDA;
+  uint8_t* ws = static_cast<uint8_t*>(workspace);
+  RescoreArgs a{};
+  a.targets = targets;
+  a.status = reinterpret_cast<uint32_t*>(ws);
+  a.zt = reinterpret_cast<float*>(ws + g.zt_off);
+  a.part = reinterpret_cast<float2*>(ws + g.part_off);
+  a.part_t = reinterpret_cast<float*>(ws + g.part_t_off);
+  a.n_tokens = n_tokens;
+  a.vocab = vocab_shard;
+  a.num_kb = g.num_kb;
+  a.num_m_ctx = g.num_m_ctx;
+  a.num_m = g.num_m;
+  a.num_vt = g.num_vt;
+  a.num_chunks = g.num_chunks;
+  a.tiles_per_chunk = g.tiles_per_chunk;
+  a.num_units = static_cast<int32_t>(ceil_div(g.num_m, cs) * g.num_chunks);
+  a.group_m = kGroupM;
+  a.target_offset = vocab_offset;
+  a.timeout_ns = kDefaultTimeoutNs;
+  cudaStream_t st = as_stream(cuda_stream);
+  if (cudaMemsetAsync(a.status, 0, sizeof(uint32_t), st) != cudaSuccess) return HDL_ERR_CUDA;
+  // rows whose target this shard does not hold keep a NaN target logit
+  if (cudaMemsetAsync(a.zt, 0xFF, static_cast<size_t>(2 * n_tokens) * sizeof(float), st) !=
+      cudaSuccess)
+    return HDL_ERR_CUDA;
+  const int sms = current_sm_count();
+  if (sms <= 0) return HDL_ERR_CUDA;
+  const hdl_status ls =
+      dt == HDL_F32 ? launch_rescore<true, kDefaultMode, true>(tm_h0, tm_h1, tm_w, a, sms, st)
+                    : launch_rescore<false, kDefaultMode, true>(tm_h0, tm_h1, tm_w, a, sms, st);
+  if (ls != HDL_OK) return ls;
+  if (launch_status() != HDL_OK) return HDL_ERR_CUDA;
+  const int64_t blocks = ceil_div(2 * n_tokens, 256);
+  const int grid = static_cast<int>(blocks < 8 * sms ? blocks : 8 * sms);
+  shard_stats_kernel<<<grid, 256, 0, st>>>(a.part, a.part_t, a.zt, n_tokens, g.num_chunks,
+                                           reinterpret_cast<float4*>(stats));
+  return launch_status();
+}
+
+extern "C" hdl_status hdl_merge_vocab_shards(const float* stats, int32_t n_shards,
+                                             int64_t n_tokens, float* logp_orig,
+                                             float* logp_hind, float* delta,
+                                             float* entropy_orig, float* entropy_hind,
+                                             void* cuda_stream) {
+  if (n_shards <= 0 || n_tokens < 0) return HDL_ERR_INVALID_ARG;
+  if (n_tokens == 0) return HDL_OK;
+  if (!stats || !logp_orig || !logp_hind) return HDL_ERR_INVALID_ARG;
+  if (!aligned_to(stats, 16) || !aligned_to(logp_orig, 4) || !aligned_to(logp_hind, 4) ||
+      (delta && !aligned_to(delta, 4)) || (entropy_orig && !aligned_to(entropy_orig, 4)) ||
+      (entropy_hind && !aligned_to(entropy_hind, 4)))
+    return HDL_ERR_INVALID_ARG;
+  const int sms = current_sm_count();
+  if (sms <= 0) return HDL_ERR_CUDA;
+  const int64_t blocks = ceil_div(n_tokens, 256);
+  const int grid = static_cast<int>(blocks < 8 * sms ? blocks : 8 * sms);
+  merge_shards_kernel<<<grid, 256, 0, as_stream(cuda_stream)>>>(
+      reinterpret_cast<const float4*>(stats), n_shards, n_tokens, logp_orig, logp_hind, delta,
+      entropy_orig, entropy_hind);
+  return launch_status();
 }

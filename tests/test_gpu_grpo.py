@@ -1,0 +1,72 @@
+"""The GRPO update after branch selection on the GPU against the oracle:
+group-relative advantages and the asymmetric-clip token-level loss and its
+gradient on suffix-only masks (Sections 3, 3.3, 4.1)."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def hdl():
+    import __graft_entry__
+    __graft_entry__.build()
+    import paper_2609_36864_gb300 as m
+    return m
+
+
+def make_batch(seed, n_groups, max_len):
+    rng = np.random.default_rng(seed)
+    sizes = rng.integers(1, 17, size=n_groups)
+    sizes[:2] = [16, 1]                               # a full group and a lone trajectory
+    goffs = np.concatenate([[0], np.cumsum(sizes)]).astype(np.int32)
+    J = int(goffs[-1])
+    lens = rng.integers(0, max_len, size=J)
+    toffs = np.concatenate([[0], np.cumsum(lens)]).astype(np.int64)
+    T = int(toffs[-1])
+    rewards = rng.random(J).astype(np.float32)
+    rewards[goffs[2]:goffs[3]] = 0.5                  # uniform rewards: zero advantage
+    lpo = (-rng.exponential(size=T)).astype(np.float32)
+    lpn = (lpo + rng.normal(scale=0.3, size=T)).astype(np.float32)   # ratios across the clip
+    mask = (rng.random(T) < 0.7).astype(np.uint8)
+    return lpn, lpo, mask, toffs, rewards, goffs
+
+
+@pytest.mark.parametrize("seed,n_groups,max_len", [(0, 40, 300), (1, 8, 5000), (2, 300, 30)])
+def test_grpo_loss_matches_oracle(hdl, seed, n_groups, max_len):
+    lpn, lpo, mask, toffs, R, goffs = make_batch(seed, n_groups, max_len)
+    t = lambda x: torch.from_numpy(x).cuda()
+    adv, grad, stats = hdl.hdl_grpo_loss(t(lpn), t(lpo), t(mask), t(toffs), t(R), t(goffs))
+    A_ref = oracle.group_advantages(R, goffs)
+    assert np.allclose(adv.cpu().numpy(), A_ref, rtol=0, atol=1e-6)
+    # the clip decision is taken in float32 on both sides (the kernel's
+    # precision); the values are compared against float64
+    loss, g_ref, (n, clip_frac, mean_r) = oracle.grpo_token_loss(
+        lpn, lpo, mask, toffs, adv.cpu().numpy().astype(np.float64), decide_in=np.float32)
+    st = stats.cpu().numpy()
+    assert st[1] == n
+    assert abs(st[0] - loss) <= 1e-5 * max(1.0, abs(loss))
+    assert abs(st[2] - clip_frac) <= 1e-6
+    assert abs(st[3] - mean_r) <= 1e-5
+    g = grad.cpu().numpy()
+    assert np.all((g == 0) == (g_ref == 0))
+    assert np.all(np.abs(g - g_ref) <= 1e-5 * np.abs(g_ref).max())
+    assert np.all(g[mask == 0] == 0)
+
+
+def test_grpo_paper_group(hdl):
+    """One problem of the paper's default layout: 2 roots + 2 x (3 + 4)
+    continuations = G = 16 (Section 4.1); equal rewards give zero loss."""
+    goffs = np.array([0, 16], np.int32)
+    lens = np.full(16, 50)
+    toffs = np.concatenate([[0], np.cumsum(lens)]).astype(np.int64)
+    R = np.full(16, 1.0, np.float32)
+    lp = np.full(800, -0.5, np.float32)
+    mask = np.ones(800, np.uint8)
+    t = lambda x: torch.from_numpy(x).cuda()
+    adv, grad, stats = hdl.hdl_grpo_loss(t(lp), t(lp), t(mask), t(toffs), t(R), t(goffs))
+    assert torch.all(adv == 0) and stats[0].item() == 0 and stats[1].item() == 800
+    assert torch.all(grad == 0)

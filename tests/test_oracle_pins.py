@@ -432,3 +432,99 @@ def test_planted_mistakes_mask():
     for mutant in (strict, ignores_valid):
         with pytest.raises(AssertionError):
             check_mask(mutant)
+
+
+
+# ------------------------------------------------------- GRPO update (next)
+def check_advantages(fn):
+    A = fn([1.0, 0.0, 0.5, 0.5, 3.0, 2.0, 2.0, 2.0], [0, 3, 5, 5, 8])
+    assert np.allclose(A, [0.5, -0.5, 0.0, -1.25, 1.25, 0.0, 0.0, 0.0], atol=1e-15)
+    rng = np.random.default_rng(1)
+    offs = np.concatenate([[0], np.cumsum(rng.integers(1, 17, size=20))])
+    R = rng.random(offs[-1])
+    A = fn(R, offs)
+    for g in range(20):
+        assert abs(A[offs[g]:offs[g + 1]].sum()) < 1e-12      # mean-centred
+    assert np.all(fn(np.ones(16), [0, 16]) == 0)              # uniform rewards: no signal
+
+
+def test_advantages():
+    check_advantages(O.group_advantages)
+
+
+def check_grpo_loss(fn):
+    # hand cases of the asymmetric clip (eps 0.2 / 0.28), one token each
+    for r, A, want in ((1.5, 1.0, 1.28), (0.5, -1.0, -0.8), (0.5, 1.0, 0.5),
+                       (1.5, -1.0, -1.5), (1.1, 2.0, 2.2), (0.7, 1.0, 0.7)):
+        loss, grad, _ = fn([math.log(r)], [0.0], [1], [0, 1], [A])
+        assert abs(loss + want) < 1e-12, (r, A, loss)
+    # ratio 1: loss = -sum_j A_j L_j / sum_j L_j over masked tokens
+    offs = [0, 3, 7, 8]
+    mask = [1, 1, 0, 1, 1, 1, 1, 0]
+    A = [1.0, -0.5, 2.0]
+    loss, grad, st = fn(np.zeros(8), np.zeros(8), mask, offs, A)
+    assert abs(loss - (-(1.0 * 2 + (-0.5) * 4) / 6)) < 1e-12 and st[0] == 6
+    assert grad[2] == 0 and grad[7] == 0                       # masked tokens carry none
+    # gradient = central finite difference of the loss (away from clip edges)
+    rng = np.random.default_rng(2)
+    n = 40
+    offs = [0, 10, 25, 40]
+    A = [0.7, -1.3, 0.4]
+    lpo = rng.normal(size=n)
+    lpn = lpo + rng.uniform(-0.5, 0.5, size=n)
+    mask = (rng.random(n) < 0.8).astype(np.uint8)
+    loss, grad, _ = fn(lpn, lpo, mask, offs, A)
+    h = 1e-6
+    for t in range(n):
+        e = np.zeros(n)
+        e[t] = h
+        lp = fn(lpn + e, lpo, mask, offs, A)[0]
+        lm = fn(lpn - e, lpo, mask, offs, A)[0]
+        fd = (lp - lm) / (2 * h)
+        r = math.exp(lpn[t] - lpo[t])
+        if abs(r - 0.8) > 1e-3 and abs(r - 1.28) > 1e-3:
+            assert abs(fd - grad[t]) < 1e-7, (t, fd, grad[t])
+    # masked tokens do not move the loss
+    lpn2 = lpn.copy()
+    lpn2[mask == 0] += 3.0
+    assert abs(fn(lpn2, lpo, mask, offs, A)[0] - loss) < 1e-15
+
+
+def test_grpo_loss():
+    check_grpo_loss(O.grpo_token_loss)
+
+
+def test_planted_mistakes_grpo():
+    def std_normalised(R, offs):
+        A = O.group_advantages(R, offs)
+        R = np.asarray(R, float)
+        for g in range(len(offs) - 1):
+            if offs[g + 1] <= offs[g]:
+                continue
+            sd = R[offs[g]:offs[g + 1]].std()
+            if sd > 0:
+                A[offs[g]:offs[g + 1]] /= sd
+        return A
+    with pytest.raises(AssertionError):
+        check_advantages(std_normalised)
+
+    def symmetric_clip(lpn, lpo, mask, offs, A):
+        return O.grpo_token_loss(lpn, lpo, mask, offs, A, 0.2, 0.2)
+
+    def sequence_mean(lpn, lpo, mask, offs, A):
+        loss, grad, st = O.grpo_token_loss(lpn, lpo, mask, offs, A)
+        m = np.asarray(mask) != 0
+        per = []
+        for j in range(len(offs) - 1):
+            s_, e_ = offs[j], offs[j + 1]
+            if m[s_:e_].any():
+                l_, _, _ = O.grpo_token_loss(lpn[s_:e_], lpo[s_:e_], mask[s_:e_],
+                                             [0, e_ - s_], [A[j]])
+                per.append(l_)
+        return float(np.mean(per)), grad, st
+
+    def no_clip(lpn, lpo, mask, offs, A):
+        return O.grpo_token_loss(lpn, lpo, mask, offs, A, 1e9, 1e9)
+    for mutant in (symmetric_clip, sequence_mean, no_clip):
+        with pytest.raises(AssertionError):
+            check_grpo_loss(mutant)
