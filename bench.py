@@ -46,6 +46,8 @@ def parse():
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu", action="store_true")
     p.add_argument("--cpu-seconds", type=float, default=12.0)
+    p.add_argument("--micro", default=None, choices=["select", "mask", "grpo"],
+                   help="bandwidth micro-benchmark of one HBM-bound kernel at a scaled size")
     return p.parse_args()
 
 
@@ -423,8 +425,79 @@ def run_gpu(args, world, rank, local):
     print(json.dumps(line), flush=True)
 
 
+def run_micro(args):
+    """GB/s of the selection, mask or loss kernel against the HBM peak, on a
+    scaled synthetic case (the benchmark workloads make them latency bound).
+    Algorithmic bytes: select N*(4+1) + 8(R+1) + R*k*(4+4) + 4R; mask
+    2*sum(L) + 12*C; grpo 13*T (pass 1) + 8*T (gradient scale) + 8*J."""
+    import paper_2609_36864_gb300 as hdl
+    from paper_2609_36864_gb300 import build as b
+    b.build()
+    g = torch.Generator(device="cuda").manual_seed(0)
+    dev = "cuda"
+    if args.micro == "select":
+        R, T, k = 8192, 4096, 8
+        N = R * T
+        delta = torch.rand(N, generator=g, device=dev)
+        valid = (torch.rand(N, generator=g, device=dev) < 0.8).to(torch.uint8)
+        offs = torch.arange(0, N + 1, T, dtype=torch.int64, device=dev)
+        bp = torch.empty((R, k), dtype=torch.int32, device=dev)
+        ns = torch.empty(R, dtype=torch.int32, device=dev)
+        bd = torch.empty((R, k), dtype=torch.float32, device=dev)
+        fn = lambda: hdl.hdl_select_branches(delta, valid, offs, k, branch_pos=bp,
+                                             n_selected=ns, branch_delta=bd)
+        nbytes = N * 5 + 8 * (R + 1) + R * k * 8 + 4 * R
+        cfg = {"roots": R, "tokens_per_root": T, "k": k}
+    elif args.micro == "mask":
+        C, L = 32768, 4096
+        offs = torch.arange(0, C * L + 1, L, dtype=torch.int64, device=dev)
+        cb = torch.randint(-1, L, (C,), generator=g, device=dev, dtype=torch.int32)
+        valid = (torch.rand(C * L, generator=g, device=dev) < 0.8).to(torch.uint8)
+        mask = torch.empty(C * L, dtype=torch.uint8, device=dev)
+        fn = lambda: hdl.hdl_suffix_mask(cb, offs, valid, mask=mask)
+        nbytes = 2 * C * L + 12 * C
+        cfg = {"continuations": C, "length": L}
+    else:
+        J, L = 16384, 4096
+        T = J * L
+        lpo = -torch.rand(T, generator=g, device=dev) * 3
+        lpn = lpo + torch.randn(T, generator=g, device=dev) * 0.3
+        m = (torch.rand(T, generator=g, device=dev) < 0.7).to(torch.uint8)
+        toffs = torch.arange(0, T + 1, L, dtype=torch.int64, device=dev)
+        R = torch.rand(J, generator=g, device=dev)
+        goffs = torch.arange(0, J + 1, 16, dtype=torch.int32, device=dev)
+        adv = torch.empty(J, dtype=torch.float32, device=dev)
+        grad = torch.empty(T, dtype=torch.float32, device=dev)
+        st = torch.empty(4, dtype=torch.float32, device=dev)
+        ws = torch.empty(hdl.hdl_grpo_loss_workspace_bytes(), dtype=torch.uint8, device=dev)
+        fn = lambda: hdl.hdl_grpo_loss(lpn, lpo, m, toffs, R, goffs, advantages=adv, grad=grad,
+                                       stats=st, workspace=ws)
+        nbytes = 13 * T + 8 * T + 8 * J
+        cfg = {"trajectories": J, "length": L, "group": 16}
+    for _ in range(max(args.warmup, 3)):
+        fn()
+    torch.cuda.synchronize()
+    evs = []
+    for _ in range(args.steps):      # inputs are larger than L2 (>= 168 MB)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        fn()
+        e1.record()
+        evs.append((e0, e1))
+    torch.cuda.synchronize()
+    ms = float(np.median([a.elapsed_time(b_) for a, b_ in evs]))
+    _, _, hbm, src = peaks()
+    gbs = nbytes / (ms / 1e3) / 1e9
+    print(json.dumps({"micro": args.micro, "config": cfg, "ms": ms, "bytes": nbytes,
+                      "achieved_gbs": gbs, "peak_gbs": hbm, "frac": gbs / hbm,
+                      "peak_kind": f"hbm copy ({src})", "steps": args.steps}), flush=True)
+
+
 def main():
     args = parse()
+    if args.micro:
+        run_micro(args)
+        return
     world, rank, local = dist_setup()
     if args.impl == "reference":
         run_reference(args, world, rank)
