@@ -429,7 +429,8 @@ def run_micro(args):
     """GB/s of the selection, mask or loss kernel against the HBM peak, on a
     scaled synthetic case (the benchmark workloads make them latency bound).
     Algorithmic bytes: select N*(4+1) + 8(R+1) + R*k*(4+4) + 4R; mask
-    2*sum(L) + 12*C; grpo 13*T (pass 1) + 8*T (gradient scale) + 8*J."""
+    2*sum(L) + 12*C; grpo 1*T (mask count) + 13*T (scores, mask, gradient)
+    + 8*J."""
     import paper_2609_36864_gb300 as hdl
     from paper_2609_36864_gb300 import build as b
     b.build()
@@ -472,7 +473,7 @@ def run_micro(args):
         ws = torch.empty(hdl.hdl_grpo_loss_workspace_bytes(), dtype=torch.uint8, device=dev)
         fn = lambda: hdl.hdl_grpo_loss(lpn, lpo, m, toffs, R, goffs, advantages=adv, grad=grad,
                                        stats=st, workspace=ws)
-        nbytes = 13 * T + 8 * T + 8 * J
+        nbytes = 14 * T + 8 * J
         cfg = {"trajectories": J, "length": L, "group": 16}
     for _ in range(max(args.warmup, 3)):
         fn()

@@ -4,6 +4,7 @@
 #include <cuda_runtime.h>
 
 #include <cstdint>
+#include <climits>
 
 #include "hdl.h"
 #include "hdl_internal.h"
@@ -86,65 +87,60 @@ __global__ void __launch_bounds__(kAssignThreads)
   }
 }
 
-// Index of the continuation holding mask byte p: the last c with
-// offs[c] <= p, searched in [0, n).
-__device__ __forceinline__ int find_cont(const int64_t* offs, int n, int64_t p) {
-  int lo = 0, hi = n - 1;
-  while (lo < hi) {
-    const int mid = (lo + hi + 1) >> 1;
-    if (offs[mid] <= p) lo = mid; else hi = mid - 1;
-  }
-  return lo;
+// 0x01 in every byte of w that is nonzero, 0x00 elsewhere.
+__device__ __forceinline__ uint32_t nonzero_bytes(uint32_t w) {
+  return (((w & 0x7F7F7F7Fu) + 0x7F7F7F7Fu) | w) >> 7 & 0x01010101u;
 }
 
-// mask byte of continuation c at absolute position p
-__device__ __forceinline__ uint8_t mask_byte(const int32_t* cb, const int64_t* offs, int c,
-                                             int64_t p, const uint8_t* valid) {
-  const int32_t b = cb[c];
-  const int64_t t = p - offs[c];
-  const bool on = b >= 0 && t >= b && (valid == nullptr || valid[p] != 0);
-  return on ? 1 : 0;
-}
-
-// Grid-stride over 16-byte chunks of [lo, hi): whole chunks are read and
-// written with 16-byte vector accesses, the two edge chunks byte by byte.
+// One warp per continuation c: bytes [s, e) = [offs[c], offs[c+1]) clipped to
+// the mask; byte p is on iff p >= thr (= s + b, or never when b < 0) and it is
+// valid.  The 16-byte-aligned body is read and written 16 bytes per lane, the
+// head and tail bytes one by one, and only the one vector that contains thr
+// is resolved byte by byte.
 template <bool kVec>
 __global__ void __launch_bounds__(kMaskThreads)
     suffix_mask_kernel(const int32_t* __restrict__ cb, const int64_t* __restrict__ offs,
                        int32_t n_cont, const uint8_t* __restrict__ valid,
                        uint8_t* __restrict__ mask, int64_t mask_len) {
-  int64_t lo = offs[0], hi = offs[n_cont];
-  lo = lo < 0 ? 0 : lo;
-  hi = hi > mask_len ? mask_len : hi;
-  if (hi <= lo) return;
-  const int64_t c0 = lo / 16, c1 = (hi + 15) / 16;
-  for (int64_t ch = c0 + blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; ch < c1;
-       ch += static_cast<int64_t>(gridDim.x) * blockDim.x) {
-    const int64_t p0 = ch * 16;
-    const int64_t first = p0 > lo ? p0 : lo;
-    int c = find_cont(offs, n_cont, first);
-    if (kVec && p0 >= lo && p0 + 16 <= hi) {
-      uint4 vv = make_uint4(0xFFFFFFFFu, 0xFFFFFFFFu, 0xFFFFFFFFu, 0xFFFFFFFFu);
-      if (valid) vv = *reinterpret_cast<const uint4*>(valid + p0);
-      const uint8_t* vb = reinterpret_cast<const uint8_t*>(&vv);
-      uint4 out;
-      uint8_t* ob = reinterpret_cast<uint8_t*>(&out);
-#pragma unroll
-      for (int i = 0; i < 16; ++i) {
-        const int64_t p = p0 + i;
-        while (c + 1 < n_cont && p >= offs[c + 1]) ++c;
-        const int32_t b = cb[c];
-        const int64_t t = p - offs[c];
-        ob[i] = (b >= 0 && t >= b && vb[i] != 0) ? 1 : 0;
-      }
-      *reinterpret_cast<uint4*>(mask + p0) = out;
-    } else {
-      const int64_t last = p0 + 16 < hi ? p0 + 16 : hi;
-      for (int64_t p = first; p < last; ++p) {
-        while (c + 1 < n_cont && p >= offs[c + 1]) ++c;
-        mask[p] = mask_byte(cb, offs, c, p, valid);
-      }
+  const int lane = threadIdx.x & 31;
+  const int64_t warps = static_cast<int64_t>(gridDim.x) * (blockDim.x / 32);
+  for (int64_t c = static_cast<int64_t>(blockIdx.x) * (blockDim.x / 32) + (threadIdx.x >> 5);
+       c < n_cont; c += warps) {
+    int64_t s = offs[c], e = offs[c + 1];
+    const int32_t b = cb[c];
+    const int64_t thr = b >= 0 ? s + b : INT64_MAX;
+    s = s < 0 ? 0 : s;
+    e = e > mask_len ? mask_len : e;
+    if (e <= s) continue;
+    int64_t h = s, body = s;
+    if (kVec) {
+      h = (s + 15) & ~int64_t{15};
+      h = h < e ? h : e;
+      body = h + ((e - h) & ~int64_t{15});
     }
+    for (int64_t p = s + lane; p < h; p += 32)
+      mask[p] = (p >= thr && (valid == nullptr || valid[p] != 0)) ? 1 : 0;
+    for (int64_t p = h + 16 * lane; p < body; p += 16 * 32) {
+      uint4 v = make_uint4(0x01010101u, 0x01010101u, 0x01010101u, 0x01010101u);
+      if (valid) {
+        v = *reinterpret_cast<const uint4*>(valid + p);
+        v.x = nonzero_bytes(v.x);
+        v.y = nonzero_bytes(v.y);
+        v.z = nonzero_bytes(v.z);
+        v.w = nonzero_bytes(v.w);
+      }
+      if (p + 16 <= thr) {
+        v = make_uint4(0u, 0u, 0u, 0u);
+      } else if (p < thr) {
+        uint8_t* vb = reinterpret_cast<uint8_t*>(&v);
+#pragma unroll
+        for (int i = 0; i < 16; ++i)
+          if (p + i < thr) vb[i] = 0;
+      }
+      *reinterpret_cast<uint4*>(mask + p) = v;
+    }
+    for (int64_t p = body + lane; p < e; p += 32)
+      mask[p] = (p >= thr && (valid == nullptr || valid[p] != 0)) ? 1 : 0;
   }
 }
 
@@ -182,9 +178,8 @@ extern "C" hdl_status hdl_suffix_mask(const int32_t* cont_branch, const int64_t*
   const bool vec = aligned_to(mask, 16) && (cont_valid == nullptr || aligned_to(cont_valid, 16));
   const int sms = current_sm_count();
   if (sms <= 0) return HDL_ERR_CUDA;
-  const int64_t chunks = ceil_div(mask_len, 16);
-  const int64_t blocks = ceil_div(chunks, kMaskThreads);
-  const int grid = static_cast<int>(blocks < 4 * sms ? (blocks > 0 ? blocks : 1) : 4 * sms);
+  const int64_t blocks = ceil_div(n_cont, kMaskThreads / 32);   // one warp per continuation
+  const int grid = static_cast<int>(blocks < 16 * sms ? blocks : 16 * sms);
   cudaStream_t st = as_stream(cuda_stream);
   if (vec)
     suffix_mask_kernel<true><<<grid, kMaskThreads, 0, st>>>(cont_branch, cont_offsets, n_cont,

@@ -3,19 +3,25 @@
 // policy-generated tokens are candidates; Section 4.4: of points too close
 // together only one is kept).
 //
-// One CTA per root.  A candidate is encoded as a 64-bit key whose order is
-// the ranking: high word = the score mapped to an order-preserving unsigned
-// integer (-0 folded onto +0), low word = ~t, so that equal scores rank the
-// lower position first.  Key 0 never occurs for a real candidate and means
-// "none".
-//   plain top-k: each thread keeps a sorted register list of its 16 best
-//     keys while streaming its strided share of the root; then k rounds of a
-//     block-wide max pick the winners, the owning thread popping its head.
-//   greedy spacing (gap_mode 0): k rounds, each a full scan for the best key
-//     not within min_gap of an accepted point (the greedy walk of the ranked
-//     list accepts exactly these points in this order).
-//   drop-lower spacing (gap_mode 1): plain top-k, then thread 0 walks the k
-//     points in rank order and keeps those not too close to a kept one.
+// A candidate is encoded as a 64-bit key whose order is the ranking: high
+// word = the score mapped to an order-preserving unsigned integer (-0 folded
+// onto +0), low word = ~t, so that equal scores rank the lower position
+// first.  Key 0 never occurs for a real candidate and means "none".
+//
+// Plain top-k (the default): select_topk_kernel streams each root with
+// 16-byte loads (4 scores + 4 validity bytes per lane) into one exact top-k
+// list per warp held across its lanes; a candidate is compared with the
+// current k-th best and only the few that beat it (about k ln(T/k) per root)
+// are inserted, cooperatively (ballot + shuffle), so no lane ever runs a
+// divergent insertion.  One warp per root when there are many roots, one
+// block of 16 warps per root (the per-warp lists merged by warp 0) when there
+// are few long ones.
+// Spacing rule (min_gap > 0): select_spacing_kernel, one CTA per root --
+//   greedy (gap_mode 0): k rounds, each a full scan for the best key not
+//     within min_gap of an accepted point (the greedy walk of the ranked
+//     list accepts exactly these points in this order);
+//   drop-lower (gap_mode 1): plain top-k, then thread 0 walks the k points
+//     in rank order and keeps those not too close to a kept one.
 #include <cuda_runtime.h>
 
 #include <cstdint>
@@ -85,7 +91,7 @@ __device__ __forceinline__ bool is_candidate(const float* delta, const uint8_t* 
 }
 
 __global__ void __launch_bounds__(kSelThreads)
-    select_branches_kernel(const float* __restrict__ delta, const uint8_t* __restrict__ valid,
+    select_spacing_kernel(const float* __restrict__ delta, const uint8_t* __restrict__ valid,
                            int64_t n_tokens, const int64_t* __restrict__ root_offsets,
                            int32_t n_roots, int32_t k, int32_t min_gap, int32_t gap_mode,
                            int32_t lo, int32_t hi, int32_t* __restrict__ branch_pos,
@@ -189,6 +195,193 @@ __global__ void __launch_bounds__(kSelThreads)
   }
 }
 
+// The warp's running top-k is distributed over its lanes: lane j < k holds
+// the j-th best key so far (0 = empty), lanes >= k hold 0.  tau = lane k-1's
+// key is the exact k-th best; a candidate must beat it to enter.
+struct WarpTopK {
+  uint64_t mine;   // this lane's entry
+  uint64_t tau;    // k-th best so far, on every lane
+  float tau_s;     // its score (-inf while the list is not full)
+};
+
+// Inverse of score_order on a key's high word.
+__device__ __forceinline__ float key_score(uint64_t key) {
+  if (key == 0ull) return -INFINITY;
+  const uint32_t u = static_cast<uint32_t>(key >> 32);
+  return __uint_as_float((u & 0x80000000u) ? (u ^ 0x80000000u) : ~u);
+}
+
+// Insert `key` (> tau, identical on every lane) into the list.
+__device__ __forceinline__ void wtk_insert(WarpTopK& w, uint64_t key, int k, int lane) {
+  const int pos = __popc(__ballot_sync(0xffffffffu, w.mine > key));
+  const uint64_t prev = __shfl_up_sync(0xffffffffu, w.mine, 1);
+  if (lane > pos) w.mine = prev;
+  if (lane == pos) w.mine = key;
+  if (lane >= k) w.mine = 0ull;
+  w.tau = __shfl_sync(0xffffffffu, w.mine, k - 1);
+  w.tau_s = key_score(w.tau);
+}
+
+// Offer each lane's candidate (score s at root position t; ok = valid): a
+// candidate whose score is below the k-th best's is rejected by one float
+// compare (it cannot beat tau); the few others get their key built (NaN
+// scores get none) and are inserted one at a time, lowest lane first, each
+// re-tested against the new tau.
+__device__ __forceinline__ void wtk_offer_key(WarpTopK& w, uint64_t key, int k, int lane) {
+  unsigned pending = __ballot_sync(0xffffffffu, key > w.tau);
+  while (pending) {
+    const int src = __ffs(pending) - 1;
+    const uint64_t cand = __shfl_sync(0xffffffffu, key, src);
+    wtk_insert(w, cand, k, lane);
+    if (lane == src) key = 0ull;
+    pending = __ballot_sync(0xffffffffu, key > w.tau);
+  }
+}
+
+__device__ __forceinline__ void wtk_offer(WarpTopK& w, float s, bool ok, int64_t t, int k,
+                                          int lane) {
+  ok = ok && s >= w.tau_s;
+  if (!__any_sync(0xffffffffu, ok)) return;
+  wtk_offer_key(w, ok && !isnan(s) ? make_key(s, t) : 0ull, k, lane);
+}
+
+// The warp streams absolute positions [a0, a1) of the root starting at
+// `start`: scalar head and tail, and a vector body walked in warp-uniform
+// steps of 4 x 32 four-position groups whose loads are all issued first.
+template <bool kVec>
+__device__ __forceinline__ void stream_range(WarpTopK& w, const float* delta, const uint8_t* valid,
+                                             int64_t start, int64_t a0, int64_t a1, int k,
+                                             int lane) {
+  if (!kVec) {
+    for (int64_t q = a0; q < a1; q += 32) {
+      const int64_t p = q + lane;
+      const bool in = p < a1;
+      wtk_offer(w, in ? delta[p] : 0.f, in && (valid == nullptr || valid[p] != 0), p - start, k,
+                lane);
+    }
+    return;
+  }
+  const int64_t h = a0 + ((4 - (a0 & 3)) & 3) < a1 ? a0 + ((4 - (a0 & 3)) & 3) : a1;
+  {
+    const int64_t p = a0 + lane;
+    const bool in = p < h;
+    wtk_offer(w, in ? delta[p] : 0.f, in && (valid == nullptr || valid[p] != 0), p - start, k,
+              lane);
+  }
+  const int64_t body = h + ((a1 - h) & ~int64_t{3});
+  constexpr int kBatch = 4;
+  for (int64_t q = h; q < body; q += 4 * 32 * kBatch) {
+    float4 d[kBatch];
+    uint32_t v[kBatch];
+#pragma unroll
+    for (int i = 0; i < kBatch; ++i) {
+      const int64_t p = q + 4 * (32 * i + lane);
+      if (p < body) {
+        d[i] = *reinterpret_cast<const float4*>(delta + p);
+        v[i] = valid ? *reinterpret_cast<const uint32_t*>(valid + p) : 0x01010101u;
+      } else {
+        d[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+        v[i] = 0u;
+      }
+    }
+#pragma unroll
+    for (int i = 0; i < kBatch; ++i) {
+      const int64_t t = q + 4 * (32 * i + lane) - start;
+      wtk_offer(w, d[i].x, (v[i] & 0xFFu) != 0, t, k, lane);
+      wtk_offer(w, d[i].y, (v[i] & 0xFF00u) != 0, t + 1, k, lane);
+      wtk_offer(w, d[i].z, (v[i] & 0xFF0000u) != 0, t + 2, k, lane);
+      wtk_offer(w, d[i].w, (v[i] & 0xFF000000u) != 0, t + 3, k, lane);
+    }
+  }
+  {
+    const int64_t p = body + lane;
+    const bool in = p < a1;
+    wtk_offer(w, in ? delta[p] : 0.f, in && (valid == nullptr || valid[p] != 0), p - start, k,
+              lane);
+  }
+}
+
+// kWarps == 1: one warp per root (8 roots per 256-thread block);
+// kWarps == 16: one 512-thread block per root, each warp a contiguous slice,
+// the 16 partial lists merged by warp 0 through shared memory.
+template <int kWarps, bool kVec>
+__global__ void __launch_bounds__(kWarps == 1 ? 256 : 32 * kWarps)
+    select_topk_kernel(const float* __restrict__ delta, const uint8_t* __restrict__ valid,
+                       int64_t n_tokens, const int64_t* __restrict__ root_offsets,
+                       int32_t n_roots, int32_t k, int32_t lo, int32_t hi,
+                       int32_t* __restrict__ branch_pos, int32_t* __restrict__ n_selected,
+                       float* __restrict__ branch_delta) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int roots_per_block = kWarps == 1 ? blockDim.x / 32 : 1;
+  const int64_t first =
+      static_cast<int64_t>(blockIdx.x) * roots_per_block + (kWarps == 1 ? warp : 0);
+  const int64_t step = static_cast<int64_t>(gridDim.x) * roots_per_block;
+  __shared__ uint64_t lists[kWarps == 1 ? 1 : kWarps][32];
+  for (int64_t r = first; r < n_roots; r += step) {
+    const int64_t start = root_offsets[r];
+    const int64_t end = root_offsets[r + 1];
+    const int64_t T = end > start ? end - start : 0;
+    const int64_t w_lo = lo > 0 ? lo : 0;
+    const int64_t w_hi = hi <= 0 ? T : (hi < T ? hi : T);
+    int64_t a0 = start + w_lo, a1 = start + w_hi;
+    if (a0 < 0) a0 = 0;
+    if (a1 > n_tokens) a1 = n_tokens;
+    WarpTopK w{0ull, 0ull, -INFINITY};
+    if (kWarps == 1) {
+      if (a1 > a0) stream_range<kVec>(w, delta, valid, start, a0, a1, k, lane);
+    } else {
+      const int64_t len = a1 > a0 ? a1 - a0 : 0;
+      const int64_t per = ((len + kWarps - 1) / kWarps + 3) & ~int64_t{3};
+      const int64_t s0 = a0 + per * warp;
+      const int64_t s1 = s0 + per < a1 ? s0 + per : a1;
+      if (s0 < s1) stream_range<kVec>(w, delta, valid, start, s0, s1, k, lane);
+      lists[warp][lane] = w.mine;
+      __syncthreads();
+      if (warp == 0) {
+        w = WarpTopK{0ull, 0ull, -INFINITY};
+        for (int i = 0; i < kWarps; ++i) wtk_offer_key(w, lists[i][lane], k, lane);
+      }
+      __syncthreads();
+      if (warp != 0) continue;
+    }
+    const int n = __popc(__ballot_sync(0xffffffffu, w.mine != 0ull));
+    if (lane < k) {
+      const int64_t o = r * k + lane;
+      if (lane < n) {
+        const int64_t t = key_pos(w.mine);
+        branch_pos[o] = static_cast<int32_t>(t);
+        if (branch_delta) branch_delta[o] = delta[start + t];
+      } else {
+        branch_pos[o] = -1;
+        if (branch_delta) branch_delta[o] = __int_as_float(0x7fc00000);
+      }
+    }
+    if (lane == 0) n_selected[r] = n;
+  }
+}
+
+template <bool kVec>
+hdl_status launch_topk(const float* delta, const uint8_t* valid, int64_t n_tokens,
+                       const int64_t* offs, int32_t n_roots, int32_t k, int32_t lo, int32_t hi,
+                       int32_t* bp, int32_t* ns, float* bd, int sms, cudaStream_t st) {
+  if (n_roots >= 2 * sms) {
+    // persistent: as many 8-warp blocks as fit at once, warps loop over roots
+    int per_sm = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, select_topk_kernel<1, kVec>, 256,
+                                                      0) != cudaSuccess || per_sm <= 0)
+      per_sm = 4;
+    const int64_t blocks = (n_roots + 7) / 8;
+    const int64_t cap = static_cast<int64_t>(per_sm) * sms;
+    const int grid = static_cast<int>(blocks < cap ? blocks : cap);
+    select_topk_kernel<1, kVec><<<grid, 256, 0, st>>>(delta, valid, n_tokens, offs, n_roots, k,
+                                                      lo, hi, bp, ns, bd);
+  } else {
+    select_topk_kernel<16, kVec><<<n_roots, 512, 0, st>>>(delta, valid, n_tokens, offs,
+                                                          n_roots, k, lo, hi, bp, ns, bd);
+  }
+  return launch_status();
+}
+
 }  // namespace
 }  // namespace hdl
 
@@ -206,6 +399,7 @@ extern "C" hdl_status hdl_select_branches(const float* delta, const uint8_t* val
   if (opts) o = *opts;
   if (o.min_gap < 0 || (o.gap_mode != 0 && o.gap_mode != 1)) return HDL_ERR_INVALID_ARG;
   if (n_roots == 0) return HDL_OK;
+  if (n_tokens >= (int64_t{1} << 31)) return HDL_ERR_UNSUPPORTED;
   if (!root_offsets || !n_selected || (k > 0 && !branch_pos) || (n_tokens > 0 && !delta))
     return HDL_ERR_INVALID_ARG;
   if (!aligned_to(root_offsets, 8) || !aligned_to(n_selected, 4) ||
@@ -214,9 +408,22 @@ extern "C" hdl_status hdl_select_branches(const float* delta, const uint8_t* val
     return HDL_ERR_INVALID_ARG;
   const int sms = current_sm_count();
   if (sms <= 0) return HDL_ERR_CUDA;
-  const int grid = n_roots < 32 * sms ? n_roots : 32 * sms;
-  select_branches_kernel<<<grid, kSelThreads, 0, as_stream(cuda_stream)>>>(
-      delta, valid, n_tokens, root_offsets, n_roots, k, o.min_gap, o.gap_mode, o.lo, o.hi,
-      branch_pos, n_selected, branch_delta);
-  return launch_status();
+  cudaStream_t st = as_stream(cuda_stream);
+  if (o.min_gap > 0) {
+    const int grid = n_roots < 32 * sms ? n_roots : 32 * sms;
+    select_spacing_kernel<<<grid, kSelThreads, 0, st>>>(
+        delta, valid, n_tokens, root_offsets, n_roots, k, o.min_gap, o.gap_mode, o.lo, o.hi,
+        branch_pos, n_selected, branch_delta);
+    return launch_status();
+  }
+  if (k == 0) {
+    if (cudaMemsetAsync(n_selected, 0, sizeof(int32_t) * n_roots, st) != cudaSuccess)
+      return HDL_ERR_CUDA;
+    return HDL_OK;
+  }
+  const bool vec = aligned_to(delta, 16) && (valid == nullptr || aligned_to(valid, 4));
+  return vec ? launch_topk<true>(delta, valid, n_tokens, root_offsets, n_roots, k, o.lo, o.hi,
+                                 branch_pos, n_selected, branch_delta, sms, st)
+             : launch_topk<false>(delta, valid, n_tokens, root_offsets, n_roots, k, o.lo, o.hi,
+                                  branch_pos, n_selected, branch_delta, sms, st);
 }

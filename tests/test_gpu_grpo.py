@@ -70,3 +70,27 @@ def test_grpo_paper_group(hdl):
     adv, grad, stats = hdl.hdl_grpo_loss(t(lp), t(lp), t(mask), t(toffs), t(R), t(goffs))
     assert torch.all(adv == 0) and stats[0].item() == 0 and stats[1].item() == 800
     assert torch.all(grad == 0)
+
+
+@pytest.mark.parametrize("shift", [1, 2, 3])
+def test_grpo_unaligned(hdl, shift):
+    """First trajectory starting at a token that is not a multiple of 4, and
+    buffers that are not 16-byte aligned: the scalar loading paths."""
+    lpn, lpo, mask, toffs, R, goffs = make_batch(10 + shift, 30, 200)
+    T = len(lpn)
+    # `shift` leading tokens outside every trajectory, carrying no loss
+    pad = lambda x, v: np.concatenate([np.full(shift, v, x.dtype), x])
+    lpn2, lpo2, mask2 = pad(lpn, -1.0), pad(lpo, -1.0), pad(mask, 0)
+    toffs2 = toffs + shift
+    buf = lambda x: torch.from_numpy(np.concatenate([x[:1], x])).cuda()[1:]   # misalign
+    adv, grad, stats = hdl.hdl_grpo_loss(buf(lpn2), buf(lpo2), buf(mask2),
+                                         torch.from_numpy(toffs2).cuda(),
+                                         torch.from_numpy(R).cuda(),
+                                         torch.from_numpy(goffs).cuda())
+    loss, g_ref, (n, cf, mr) = oracle.grpo_token_loss(
+        lpn, lpo, mask, toffs, adv.cpu().numpy().astype(np.float64), decide_in=np.float32)
+    st = stats.cpu().numpy()
+    assert st[1] == n and abs(st[0] - loss) <= 1e-5 * max(1.0, abs(loss))
+    g = grad.cpu().numpy()
+    assert np.all(g[:shift] == 0)
+    assert np.all(np.abs(g[shift:] - g_ref) <= 1e-5 * np.abs(g_ref).max())

@@ -48,6 +48,9 @@ def assert_select_equal(hdl, delta, valid, offs, k, **kw):
 
 
 CASES = [
+    (list(np.random.default_rng(5).integers(0, 300, size=700)), 8, {}),   # warp per root
+    (list(np.random.default_rng(6).integers(0, 70, size=400)), 16, {}),
+    (list(np.random.default_rng(7).integers(0, 900, size=350)), 3, {}),
     ([0, 1, 2, 3, 17, 100, 511, 513, 4096], 4, {}),
     ([16384, 16384, 12000], 16, {}),                       # maximum k, long roots
     ([3, 5, 1, 0, 2], 8, {}),                              # k > T
@@ -182,3 +185,18 @@ def test_suffix_mask_unaligned_and_offset_range(hdl):
         lo = shift
         assert np.all(got[:lo] == 7) and np.all(got[lo + total:] == 7)
         assert np.array_equal(got[lo:lo + total], ref)
+
+
+@pytest.mark.parametrize("n_roots", [5, 600])
+def test_select_unaligned_buffers(hdl, n_roots):
+    """Scores / validity not 16- / 4-byte aligned: the scalar loading path."""
+    lengths = list(np.random.default_rng(n_roots).integers(0, 500, size=n_roots))
+    delta, valid, offs = make_roots(lengths, 12, tie_levels=5)
+    N = len(delta)
+    d = torch.zeros(N + 1, dtype=torch.float32, device="cuda")
+    v = torch.zeros(N + 1, dtype=torch.uint8, device="cuda")
+    d[1:] = torch.from_numpy(delta).cuda()
+    v[1:] = torch.from_numpy(valid).cuda()
+    bp, ns, bd = hdl.hdl_select_branches(d[1:], v[1:], torch.from_numpy(offs).cuda(), 8)
+    pos, nsel, val = oracle.select_branches(delta.astype(np.float64), valid, offs, 8)
+    assert np.array_equal(ns.cpu().numpy(), nsel) and np.array_equal(bp.cpu().numpy(), pos)
