@@ -302,8 +302,8 @@ __device__ __forceinline__ void stream_range(WarpTopK& w, const float* delta, co
 }
 
 // kWarps == 1: one warp per root (8 roots per 256-thread block);
-// kWarps == 16: one 512-thread block per root, each warp a contiguous slice,
-// the 16 partial lists merged by warp 0 through shared memory.
+// kWarps == 16: one block per root, each warp a contiguous slice, the
+// partial lists merged by warp 0 through shared memory.
 template <int kWarps, bool kVec>
 __global__ void __launch_bounds__(kWarps == 1 ? 256 : 32 * kWarps)
     select_topk_kernel(const float* __restrict__ delta, const uint8_t* __restrict__ valid,
@@ -360,12 +360,15 @@ __global__ void __launch_bounds__(kWarps == 1 ? 256 : 32 * kWarps)
   }
 }
 
+// Many roots: one warp per root, a persistent grid of as many 8-warp blocks
+// as are resident at once.  Few roots: 16 warps per root so that the GPU
+// fills.  (Splitting mid-length roots over 4 warps was measured slower: the
+// per-root barrier and merge cost more than the shorter chains save.)
 template <bool kVec>
 hdl_status launch_topk(const float* delta, const uint8_t* valid, int64_t n_tokens,
                        const int64_t* offs, int32_t n_roots, int32_t k, int32_t lo, int32_t hi,
                        int32_t* bp, int32_t* ns, float* bd, int sms, cudaStream_t st) {
   if (n_roots >= 2 * sms) {
-    // persistent: as many 8-warp blocks as fit at once, warps loop over roots
     int per_sm = 0;
     if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, select_topk_kernel<1, kVec>, 256,
                                                       0) != cudaSuccess || per_sm <= 0)

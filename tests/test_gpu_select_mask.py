@@ -51,6 +51,8 @@ CASES = [
     (list(np.random.default_rng(5).integers(0, 300, size=700)), 8, {}),   # warp per root
     (list(np.random.default_rng(6).integers(0, 70, size=400)), 16, {}),
     (list(np.random.default_rng(7).integers(0, 900, size=350)), 3, {}),
+    (list(np.random.default_rng(8).integers(1024, 3000, size=330)), 8, {}),   # 4 warps / root
+    (list(np.random.default_rng(9).integers(8192, 8800, size=310)), 5, {}),   # 16 warps / root
     ([0, 1, 2, 3, 17, 100, 511, 513, 4096], 4, {}),
     ([16384, 16384, 12000], 16, {}),                       # maximum k, long roots
     ([3, 5, 1, 0, 2], 8, {}),                              # k > T
