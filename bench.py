@@ -307,29 +307,39 @@ def run_gpu(args, world, rank, local):
     code, raw = hdl.hdl_device_status(path.ws, stream)
     assert code == hdl.HDL_OK, (code, raw)
 
-    # ---- kernel-only: inputs resident in HBM, larger than L2
+    # ---- kernel-only: inputs resident in HBM.  When they are larger than
+    # twice the L2 the steps run back to back; otherwise L2 is flushed (a
+    # 512 MiB write) before every step and only the steps are timed.
+    flush = None if in_bytes > 2 * L2_BYTES else torch.empty(512 << 20, dtype=torch.uint8,
+                                                            device=dev)
     ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
           for _ in range(args.steps)]
+    st_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+             for _ in range(args.steps)]
     clocks = ClockSampler(local)
     barrier(world)
     torch.cuda.synchronize()
     clocks.start()
-    t_start = torch.cuda.Event(enable_timing=True)
-    t_end = torch.cuda.Event(enable_timing=True)
-    t_start.record(stream)
     for i in range(args.steps):
+        if flush is not None:
+            flush.fill_(i & 0xFF)
+        st_ev[i][0].record(stream)
         ev[i][0].record(stream)
         path.rescore(stream)
         ev[i][1].record(stream)
         path.downstream(stream)
-    t_end.record(stream)
+        st_ev[i][1].record(stream)
     torch.cuda.synchronize()
     clk = clocks.stop()
     barrier(world)
     code, raw = hdl.hdl_device_status(path.ws, stream)
     assert code == hdl.HDL_OK, (code, raw)
-    total_ms = max_over_ranks(t_start.elapsed_time(t_end), world)
+    total_ms = max_over_ranks(float(sum(a.elapsed_time(b_) for a, b_ in st_ev)), world)
     rescore_ms = float(np.mean([a.elapsed_time(b_) for a, b_ in ev]))
+    l2_note = (f"inputs larger than L2 ({in_bytes / 2**30:.2f} GiB resident), steps back to back"
+               if flush is None else
+               f"L2 flushed before every step (inputs {in_bytes / 2**20:.1f} MiB < 2 x L2); "
+               "only the steps are timed")
     value = aggregate_value(world, N, args.steps, total_ms)
 
     # ---- end to end: every step's inputs are copied host -> device from
@@ -410,7 +420,7 @@ def run_gpu(args, world, rank, local):
         "config": {"workload": spec.name, "n_tokens": N, "d": d, "vocab": V,
                    "roots": spec.n_roots, "k": spec.k, "conts": path.C,
                    "context_rows_per_step": 2 * N,
-                   "l2": f"inputs larger than L2 ({in_bytes / 2**30:.2f} GiB resident)"},
+                   "l2": l2_note},
         "tflops": flops * args.steps / (total_ms / 1e3) / 1e12,
         "pct_bf16_peak": 100.0 * (flops * args.steps / (total_ms / 1e3) / 1e12) / burst,
         "roofline": {"bound": "tensor", "kernel": "rescore_lse_kernel (+ merge)",
