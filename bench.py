@@ -44,6 +44,9 @@ def parse():
                    help="tiny | math | code | agent | sweep_V<vocab>_N<tokens>")
     p.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
     p.add_argument("--no-e2e", action="store_true")
+    p.add_argument("--graph", action="store_true",
+                   help="capture one step in a CUDA graph and time its replays "
+                        "(for launch-bound workloads such as tiny)")
     p.add_argument("--no-cpu", action="store_true")
     p.add_argument("--cpu-seconds", type=float, default=12.0)
     p.add_argument("--micro", default=None, choices=["select", "mask", "grpo"],
@@ -288,7 +291,7 @@ def run_reference(args, world, rank):
 def run_gpu(args, world, rank, local):
     import paper_2609_36864_gb300 as hdl
     from paper_2609_36864_gb300 import build as b
-    if rank == 0 or not b.up_to_date():
+    if rank == 0:          # one rank builds; the others wait, then load it
         b.build()
     barrier(world)
     spec = spec_for(args.workload, seed=rank)
@@ -320,14 +323,31 @@ def run_gpu(args, world, rank, local):
     barrier(world)
     torch.cuda.synchronize()
     clocks.start()
+    graph = None
+    if args.graph:
+        # every call of the step is capture-safe: launches and one memset
+        side = torch.cuda.Stream()
+        side.wait_stream(stream)
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.stream(side):
+            with torch.cuda.graph(graph, stream=side):
+                path.rescore(side)
+                path.downstream(side)
+        stream.wait_stream(side)
+        graph.replay()
+        torch.cuda.synchronize()
     for i in range(args.steps):
         if flush is not None:
             flush.fill_(i & 0xFF)
         st_ev[i][0].record(stream)
         ev[i][0].record(stream)
-        path.rescore(stream)
-        ev[i][1].record(stream)
-        path.downstream(stream)
+        if graph is not None:
+            graph.replay()
+            ev[i][1].record(stream)
+        else:
+            path.rescore(stream)
+            ev[i][1].record(stream)
+            path.downstream(stream)
         st_ev[i][1].record(stream)
     torch.cuda.synchronize()
     clk = clocks.stop()
@@ -418,6 +438,7 @@ def run_gpu(args, world, rank, local):
         "vs_baseline": None, "dtype": "bf16" if spec.dtype == "bf16" else "f32",
         "data": "synthetic",
         "config": {"workload": spec.name, "n_tokens": N, "d": d, "vocab": V,
+                   "launch": "CUDA graph replay of one step" if args.graph else "eager",
                    "roots": spec.n_roots, "k": spec.k, "conts": path.C,
                    "context_rows_per_step": 2 * N,
                    "l2": l2_note},
