@@ -73,8 +73,9 @@ HDL_API const char* hdl_status_string(hdl_status s);
  *   w_lmhead        [vocab, d] row-major LM head (nn.Linear layout), type `dt`,
  *                   16-byte aligned; shared by both contexts.
  *   dt              HDL_BF16: bf16 inputs, bf16 x bf16 products with fp32
- *                   accumulation on the tensor cores.  HDL_F32: fp32 inputs,
- *                   tf32 x tf32 products with fp32 accumulation.
+ *                   accumulation on the tensor cores.  HDL_F32: fp32 inputs
+ *                   rounded to tf32 (to nearest), tf32 x tf32 products with
+ *                   fp32 accumulation.
  *   targets         [n_tokens] int32 token ids y_t in [0, vocab).
  *   n_tokens        N >= 0 tokens per context (N == 0: returns HDL_OK, no launch).
  *   d               hidden size; a positive multiple of 64, at most 65536.

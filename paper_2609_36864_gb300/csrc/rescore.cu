@@ -612,7 +612,11 @@ bool make_operand_map(CUtensorMap* m, const void* ptr, int64_t rows, int32_t d, 
   cuuint32_t box[2] = {static_cast<cuuint32_t>(kRowBytes / esize),
                        static_cast<cuuint32_t>(box_rows)};
   cuuint32_t estr[2] = {1, 1};
-  const CUresult r = enc(m, esize == 2 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT32,
+  // fp32 operands are loaded as TFLOAT32: the copy rounds them to tf32 to
+  // nearest (measured: 4.7x smaller log-prob error than letting the tensor
+  // core drop the low mantissa bits of FLOAT32 data, and no bias)
+  const CUresult r = enc(m, esize == 2 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16
+                                       : CU_TENSOR_MAP_DATA_TYPE_TFLOAT32,
                          2, const_cast<void*>(ptr), dims, strides, box, estr,
                          CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
                          CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
