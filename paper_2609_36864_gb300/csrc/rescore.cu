@@ -13,7 +13,7 @@
 // per row; a second, tiny kernel merges the chunks, forms both log-probs and
 // |Delta|.  Splitting the vocabulary keeps the set of tiles that the ~150
 // concurrently running units touch small enough to stay in L2 (grouped
-// rasterisation: kGroupM M-tiles x a few chunks at a time), instead of every
+// rasterisation: 32 M-tiles x a few chunks at a time), instead of every
 // CTA streaming its own 128 x d slice of H for the whole vocabulary.
 //
 // Roles inside a CTA of 192 threads:
@@ -50,7 +50,7 @@ constexpr int kRowBytes = 128;       // K bytes per stage (one 128-byte swizzle 
 constexpr int kMaxTilesPerChunk = 16;  // up to 4096 vocabulary entries per unit
 constexpr int64_t kMinUnits = 1216;     // 8 x 152: chunks shrink until this many units
 #ifndef HDL_GROUP_M
-#define HDL_GROUP_M 16
+#define HDL_GROUP_M 32
 #endif
 constexpr int kGroupM = HDL_GROUP_M; // M-tiles per rasterisation group (even)
 constexpr int kDefaultMode = 1;      // CTA organisation, see Cfg
@@ -677,6 +677,17 @@ int rescore_mode() {
   return mode;
 }
 
+// M-tiles per rasterisation group: HDL_GROUP_M (an even number in [2, 512])
+// overrides kGroupM for tuning; results do not depend on it.
+int rescore_group_m() {
+  static const int g = [] {
+    const char* e = std::getenv("HDL_GROUP_M");
+    const int v = e ? std::atoi(e) : 0;
+    return (v >= 2 && v <= 512 && v % 2 == 0) ? v : kGroupM;
+  }();
+  return g;
+}
+
 hdl_status check_shape(int64_t n_tokens, int32_t d, int32_t vocab, hdl_dtype dt) {
   if (n_tokens < 0 || d <= 0 || vocab <= 0) return HDL_ERR_INVALID_ARG;
   if (dt != HDL_BF16 && dt != HDL_F32) return HDL_ERR_INVALID_ARG;
@@ -757,7 +768,7 @@ extern "C" hdl_status hdl_rescore_ex(const void* h_orig, const void* h_hind,
   a.num_chunks = g.num_chunks;
   a.tiles_per_chunk = g.tiles_per_chunk;
   a.num_units = static_cast<int32_t>(ceil_div(g.num_m, cs) * g.num_chunks);
-  a.group_m = kGroupM;
+  a.group_m = rescore_group_m();
   a.inject = o.fault_inject;
   a.timeout_ns = o.wait_timeout_ns ? o.wait_timeout_ns : kDefaultTimeoutNs;
 
@@ -906,7 +917,7 @@ extern "C" hdl_status hdl_rescore_shard(const void* h_orig, const void* h_hind,
   a.num_chunks = g.num_chunks;
   a.tiles_per_chunk = g.tiles_per_chunk;
   a.num_units = static_cast<int32_t>(ceil_div(g.num_m, cs) * g.num_chunks);
-  a.group_m = kGroupM;
+  a.group_m = rescore_group_m();
   a.target_offset = vocab_offset;
   a.timeout_ns = kDefaultTimeoutNs;
   cudaStream_t st = as_stream(cuda_stream);
