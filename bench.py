@@ -72,20 +72,32 @@ def peaks():
     return 1900.0, 1700.0, 6800.0, "fallback"
 
 
+def kernel_source_digest() -> str:
+    """sha256 (16 hex digits) of the re-scoring kernel's sources with comments
+    and whitespace removed: what a DRAM-traffic record was measured on."""
+    import hashlib
+    import re
+    csrc = os.path.join(ROOT, "paper_2609_36864_gb300", "csrc")
+    h = hashlib.sha256()
+    for f in ("rescore.cu", "ptx_sm103.cuh"):
+        text = open(os.path.join(csrc, f)).read()
+        text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+        text = re.sub(r"//[^\n]*", "", text)
+        h.update(re.sub(r"\s+", "", text).encode())
+    return h.hexdigest()[:16]
+
+
 def committed_traffic(workload: str):
     """DRAM bytes per launch of the re-scoring kernel from the committed ncu
-    summary, or None if the kernel sources changed since it was taken."""
-    import hashlib
+    summary, or None if the kernel's code changed since it was taken."""
     prof = os.path.join(ROOT, "profiles", "rescore_lse_traffic.md")
-    csrc = os.path.join(ROOT, "paper_2609_36864_gb300", "csrc")
     if not os.path.exists(prof):
         return None
-    h = [hashlib.sha256(open(os.path.join(csrc, f), "rb").read()).hexdigest()[:16]
-         for f in ("rescore.cu", "ptx_sm103.cuh")]
+    digest = kernel_source_digest()
     for line in open(prof):
         f = [x.strip() for x in line.strip().strip("|").split("|")]
-        if len(f) >= 5 and f[0] == workload and f[1:3] == h:
-            return float(f[3]) + float(f[4])
+        if len(f) >= 4 and f[0] == workload and f[1] == digest:
+            return float(f[2]) + float(f[3])
     return None
 
 

@@ -10,13 +10,14 @@
 //
 // Work unit = (M-tile of 128 rows of one context, vocabulary chunk of
 // up to 16 256-wide tiles).  Each unit writes one partial (max, sum)
-// per row; a second, tiny kernel merges the chunks, forms both log-probs and
-// |Delta|.  Splitting the vocabulary keeps the set of tiles that the ~150
+// per row; a second, tiny kernel merges the chunks, forms both log-probs,
+// |Delta| and, when asked, the entropies.  Splitting the vocabulary keeps the set of tiles that the ~150
 // concurrently running units touch small enough to stay in L2 (grouped
 // rasterisation: 32 M-tiles x a few chunks at a time), instead of every
 // CTA streaming its own 128 x d slice of H for the whole vocabulary.
 //
-// Roles inside a CTA of 192 threads:
+// Roles inside a CTA of 192 threads (shown for the single-CTA organisation;
+// Cfg below describes the CTA-pair ones, the default):
 //   warp 0      TMA producer: H tile (128 x 128 B) + W tile (256 x 128 B) per
 //               K step into a kStages-deep shared-memory ring;
 //   warp 1      TMEM allocator and MMA issuer (one thread): 4 x
@@ -24,8 +25,8 @@
 //               256-column TMEM buffers so the epilogue of tile j overlaps
 //               the MMAs of tile j+1;
 //   warps 2..5  epilogue: one accumulator row per thread (TMEM lane), 32
-//               columns per tcgen05.ld, online log-sum-exp in base 2 and the
-//               target-column select.
+//               columns per tcgen05.ld, online log-sum-exp in base 2 (and the
+//               entropy numerator when asked) and the target-column select.
 #include <cuda.h>
 #include <cuda_runtime.h>
 #include <cudaTypedefs.h>
@@ -154,12 +155,6 @@ __device__ __forceinline__ void lse_fold(const float (&x)[32], float& m2, float&
   m2 = m_new;
 }
 
-// One persistent kernel for both contexts.  See Cfg for the three CTA
-// organisations.  In the cluster modes a stage may be refilled only once the
-// MMAs of the pair are done with it (mode 1: both CTAs' commits arrive on the
-// stage's empty barrier in both CTAs; mode 2: the even CTA's pair-MMA commit
-// arrives in both), and in mode 2 both CTAs' copies are counted on the even
-// CTA's full barrier and both epilogues release TMEM to the even CTA.
 // As lse_fold, also folding t = sum 2^(z log2e - m2) * z (the numerator of
 // E_p[z], for the entropy log Z - E_p[z]).
 __device__ __forceinline__ void lse_fold_ent(const float (&x)[32], float& m2, float& s,
@@ -185,6 +180,12 @@ __device__ __forceinline__ void lse_fold_ent(const float (&x)[32], float& m2, fl
   m2 = m_new;
 }
 
+// One persistent kernel for both contexts.  See Cfg for the three CTA
+// organisations.  In the cluster modes a stage may be refilled only once the
+// MMAs of the pair are done with it (mode 1: both CTAs' commits arrive on the
+// stage's empty barrier in both CTAs; mode 2: the even CTA's pair-MMA commit
+// arrives in both), and in mode 2 both CTAs' copies are counted on the even
+// CTA's full barrier and both epilogues release TMEM to the even CTA.
 template <bool kTf32, int M, bool kEnt>
 __global__ void __launch_bounds__(kThreads, 1)
     rescore_lse_kernel(const __grid_constant__ CUtensorMap tm_h0,
