@@ -104,8 +104,8 @@ __global__ void __launch_bounds__(kThreads)
 }
 
 // Per-thread running sums in fp32 (a thread sees a few hundred tokens; the
-// GPU's fp64 rate is far too low for a double add per token); the block and
-// grid folds are in double.
+// GPU's fp64 rate is far too low for a double add per token); the block fold
+// is in fp32 too, the grid fold in double.
 struct TokenOut {
   float obj, clipped, ratio;
 };
@@ -124,7 +124,7 @@ __device__ __forceinline__ float token_grad(float lpn, float lpo, float A, float
 
 // One warp per trajectory (warps loop over trajectories): the advantage is a
 // warp-uniform scalar, the trajectory's tokens are streamed with 16-byte
-// loads, four groups per lane in flight.
+// loads, two 4-token groups per lane in flight (more would cost occupancy).
 template <bool kVec>
 __global__ void __launch_bounds__(kThreads, 4)
     grpo_token_kernel(const float* __restrict__ lpn, const float* __restrict__ lpo,

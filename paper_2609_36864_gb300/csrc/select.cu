@@ -77,11 +77,6 @@ __device__ __forceinline__ uint64_t block_max_u64(uint64_t v, uint64_t* red) {
   return r;
 }
 
-struct RootView {
-  int64_t start;   // absolute index of the root's first token
-  int64_t w_lo, w_hi;  // candidate window, root-relative
-};
-
 __device__ __forceinline__ bool is_candidate(const float* delta, const uint8_t* valid,
                                              int64_t n_tokens, int64_t abs_t, float& s) {
   if (abs_t < 0 || abs_t >= n_tokens) return false;
