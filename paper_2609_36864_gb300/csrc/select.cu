@@ -9,13 +9,17 @@
 // first.  Key 0 never occurs for a real candidate and means "none".
 //
 // Plain top-k (the default): select_topk_kernel streams each root with
-// 16-byte loads (4 scores + 4 validity bytes per lane) into one exact top-k
-// list per warp held across its lanes; a candidate is compared with the
-// current k-th best and only the few that beat it (about k ln(T/k) per root)
-// are inserted, cooperatively (ballot + shuffle), so no lane ever runs a
-// divergent insertion.  One warp per root when there are many roots, one
-// block of 16 warps per root (the per-warp lists merged by warp 0) when there
-// are few long ones.
+// 16-byte loads (4 scores + 4 validity bytes per lane, a batch of 512
+// positions per warp) into one exact top-k list per warp held across its
+// lanes.  The first batch of a slice sets a floor on the k-th best score (the
+// k-th largest of the 32 lane maxima); after that a batch costs a max over
+// each lane's 16 scores and one warp vote unless some score reaches the
+// threshold.  The few candidates that beat the current k-th best (about
+// k ln(T/k) per root) are inserted one after the other (ballot + shift), or,
+// when many arrive together, by a bitonic sort of the warp's 32 candidates
+// and a bitonic merge with the list.  Many roots: S warps per root (usually
+// 1) in a persistent grid; few roots: 16 warps per root; the partial lists
+// of a root's warps are merged pairwise, a bitonic merge per level.
 // Spacing rule (min_gap > 0): select_spacing_kernel, one CTA per root --
 //   greedy (gap_mode 0): k rounds, each a full scan for the best key not
 //     within min_gap of an accepted point (the greedy walk of the ranked
@@ -25,6 +29,7 @@
 #include <cuda_runtime.h>
 
 #include <cstdint>
+#include <cstdlib>
 
 #include "hdl.h"
 #include "hdl_internal.h"
@@ -196,7 +201,8 @@ __global__ void __launch_bounds__(kSelThreads)
 struct WarpTopK {
   uint64_t mine;   // this lane's entry
   uint64_t tau;    // k-th best so far, on every lane
-  float tau_s;     // its score (-inf while the list is not full)
+  float tau_s;     // score a candidate must reach: max(tau's score, floor)
+  float floor;     // a lower bound on the final k-th best score (-inf: none)
 };
 
 // Inverse of score_order on a key's high word.
@@ -206,113 +212,256 @@ __device__ __forceinline__ float key_score(uint64_t key) {
   return __uint_as_float((u & 0x80000000u) ? (u ^ 0x80000000u) : ~u);
 }
 
-// Insert `key` (> tau, identical on every lane) into the list.
-__device__ __forceinline__ void wtk_insert(WarpTopK& w, uint64_t key, int k, int lane) {
-  const int pos = __popc(__ballot_sync(0xffffffffu, w.mine > key));
-  const uint64_t prev = __shfl_up_sync(0xffffffffu, w.mine, 1);
-  if (lane > pos) w.mine = prev;
-  if (lane == pos) w.mine = key;
-  if (lane >= k) w.mine = 0ull;
+// Bitonic network over the warp, one 64-bit key per lane.  One
+// compare-exchange with the lane `stride` away: the lower lane of the pair
+// keeps the larger key when keep_max.
+__device__ __forceinline__ uint64_t cmpx(uint64_t x, int stride, bool keep_max) {
+  const uint64_t y = __shfl_xor_sync(0xffffffffu, x, stride);
+  return keep_max == (x > y) ? x : y;
+}
+
+// Sort the warp's 32 keys into descending lane order.
+__device__ __forceinline__ uint64_t warp_sort_desc(uint64_t x, int lane) {
+#pragma unroll
+  for (int size = 2; size <= 32; size <<= 1)
+#pragma unroll
+    for (int stride = size >> 1; stride > 0; stride >>= 1) {
+      // blocks of `size` lanes alternate descending / ascending, so that
+      // each pair of neighbouring blocks forms a bitonic sequence
+      const bool desc = (lane & size) == 0;
+      const bool lower = (lane & stride) == 0;
+      x = cmpx(x, stride, lower == desc);
+    }
+  return x;
+}
+
+// Merge two descending lists of at most 16 keys, a (in lanes 0..15) and b
+// (lane j of b_rev holds b[31 - j], so lanes 16..31 read b reversed): the
+// 32 values form a bitonic sequence and five half-cleaner steps sort it.
+// Returns the merged list, descending, in lanes 0..31.
+__device__ __forceinline__ uint64_t bitonic_merge16(uint64_t a, uint64_t b_rev, int lane) {
+  uint64_t x = lane < 16 ? a : b_rev;
+#pragma unroll
+  for (int stride = 16; stride > 0; stride >>= 1) x = cmpx(x, stride, (lane & stride) == 0);
+  return x;
+}
+
+__device__ __forceinline__ void wtk_set(WarpTopK& w, uint64_t merged, int k, int lane) {
+  w.mine = lane < k ? merged : 0ull;
   w.tau = __shfl_sync(0xffffffffu, w.mine, k - 1);
-  w.tau_s = key_score(w.tau);
+  w.tau_s = fmaxf(key_score(w.tau), w.floor);
+}
+
+// Offer one key per lane (0 = none): the keys that beat the k-th best are
+// inserted -- one after the other in lane order when there are few, by
+// sorting the warp's keys and merging the top 16 with the list when there
+// are many.  In the one-by-one case no key is re-tested after an insertion:
+// inserting a key that no longer beats the k-th best changes nothing (its
+// slot is k, which is cleared), so the candidates' shuffles do not wait on
+// the list and the chain per insertion is one ballot and one shift.
+constexpr int kBulkMin = 12;
+
+__device__ __forceinline__ void wtk_offer_key(WarpTopK& w, uint64_t key, int k, int lane) {
+  unsigned pending = __ballot_sync(0xffffffffu, key > w.tau);
+  if (!pending) return;
+  if (__popc(pending) >= kBulkMin) {
+    const uint64_t c = warp_sort_desc(key > w.tau ? key : 0ull, lane);
+    const uint64_t c_rev = __shfl_sync(0xffffffffu, c, 31 - lane);
+    wtk_set(w, bitonic_merge16(w.mine, c_rev, lane), k, lane);
+    return;
+  }
+  do {
+    const int src = __ffs(pending) - 1;
+    pending &= pending - 1u;
+    const uint64_t cand = __shfl_sync(0xffffffffu, key, src);
+    const int pos = __popc(__ballot_sync(0xffffffffu, w.mine > cand));
+    const uint64_t prev = __shfl_up_sync(0xffffffffu, w.mine, 1);
+    if (lane > pos) w.mine = prev;
+    if (lane == pos) w.mine = cand;
+    if (lane >= k) w.mine = 0ull;
+  } while (pending);
+  w.tau = __shfl_sync(0xffffffffu, w.mine, k - 1);
+  w.tau_s = fmaxf(key_score(w.tau), w.floor);
 }
 
 // Offer each lane's candidate (score s at root position t; ok = valid): a
-// candidate whose score is below the k-th best's is rejected by one float
-// compare (it cannot beat tau); the few others get their key built (NaN
-// scores get none) and are inserted one at a time, lowest lane first, each
-// re-tested against the new tau.
-__device__ __forceinline__ void wtk_offer_key(WarpTopK& w, uint64_t key, int k, int lane) {
-  unsigned pending = __ballot_sync(0xffffffffu, key > w.tau);
-  while (pending) {
-    const int src = __ffs(pending) - 1;
-    const uint64_t cand = __shfl_sync(0xffffffffu, key, src);
-    wtk_insert(w, cand, k, lane);
-    if (lane == src) key = 0ull;
-    pending = __ballot_sync(0xffffffffu, key > w.tau);
-  }
-}
-
+// candidate whose score is below the k-th best's cannot beat it and is
+// rejected by the float compare alone; the others get their key built (NaN
+// scores never pass the compare).
 __device__ __forceinline__ void wtk_offer(WarpTopK& w, float s, bool ok, int64_t t, int k,
                                           int lane) {
   ok = ok && s >= w.tau_s;
   if (!__any_sync(0xffffffffu, ok)) return;
-  wtk_offer_key(w, ok && !isnan(s) ? make_key(s, t) : 0ull, k, lane);
+  wtk_offer_key(w, ok ? make_key(s, t) : 0ull, k, lane);
+}
+
+// One warp-wide batch of the vector body: kBatch groups of 32 x 4
+// consecutive positions (16 bytes of scores and 4 validity bytes per lane
+// per group); positions at or past `body` read as invalid.
+constexpr int kBatch = 4;
+constexpr int32_t kSpan = 4 * 32 * kBatch;   // positions per batch
+
+struct Batch {
+  float4 d[kBatch];
+  uint32_t v[kBatch];
+};
+
+// Positions are int32 inside the streaming loops (the entry point rejects
+// n_tokens >= 2^31).  A full batch (q + kSpan <= body) loads unguarded.
+template <bool kFull>
+__device__ __forceinline__ void load_batch(Batch& b, const float* delta, const uint8_t* valid,
+                                           int32_t q, int32_t body, int lane) {
+#pragma unroll
+  for (int i = 0; i < kBatch; ++i) {
+    const int32_t p = q + 4 * (32 * i + lane);
+    if (kFull || p < body) {
+      b.d[i] = *reinterpret_cast<const float4*>(delta + p);
+      b.v[i] = valid ? *reinterpret_cast<const uint32_t*>(valid + p) : 0x01010101u;
+    } else {
+      b.d[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+      b.v[i] = 0u;
+    }
+  }
+}
+
+// Examine a batch whose first position is q (absolute; root position =
+// absolute - start).  The common case costs a max over the lane's 16 scores
+// and one vote: no score reaches the threshold, so nothing can enter.
+// Otherwise the lanes' passing valid candidates are offered in rounds, each
+// lane its next one per round, until no lane has any left.
+__device__ __forceinline__ void offer_batch(WarpTopK& w, const Batch& b, int32_t q,
+                                            int32_t start, int k, int lane) {
+  float mx = -INFINITY;   // fmaxf ignores NaN scores
+#pragma unroll
+  for (int i = 0; i < kBatch; ++i)
+    mx = fmaxf(mx, fmaxf(fmaxf(b.d[i].x, b.d[i].y), fmaxf(b.d[i].z, b.d[i].w)));
+  if (!__any_sync(0xffffffffu, mx >= w.tau_s)) return;
+  uint32_t pass = 0;   // bit 4i+c: component c of group i
+#pragma unroll
+  for (int i = 0; i < kBatch; ++i) {
+    pass |= static_cast<uint32_t>((b.v[i] & 0xFFu) != 0 && b.d[i].x >= w.tau_s) << (4 * i);
+    pass |= static_cast<uint32_t>((b.v[i] & 0xFF00u) != 0 && b.d[i].y >= w.tau_s) << (4 * i + 1);
+    pass |= static_cast<uint32_t>((b.v[i] & 0xFF0000u) != 0 && b.d[i].z >= w.tau_s)
+            << (4 * i + 2);
+    pass |= static_cast<uint32_t>((b.v[i] & 0xFF000000u) != 0 && b.d[i].w >= w.tau_s)
+            << (4 * i + 3);
+  }
+  while (__any_sync(0xffffffffu, pass != 0)) {
+    const int j = pass ? __ffs(pass) - 1 : -1;
+    pass &= pass - 1u;
+    float sj = -INFINITY;
+#pragma unroll
+    for (int i = 0; i < kBatch; ++i) {
+      sj = j == 4 * i ? b.d[i].x : sj;
+      sj = j == 4 * i + 1 ? b.d[i].y : sj;
+      sj = j == 4 * i + 2 ? b.d[i].z : sj;
+      sj = j == 4 * i + 3 ? b.d[i].w : sj;
+    }
+    const int32_t t = q + 4 * (32 * (j >> 2) + lane) + (j & 3) - start;
+    wtk_offer_key(w, j >= 0 && sj >= w.tau_s ? make_key(sj, t) : 0ull, k, lane);
+  }
+}
+
+// Sort 32 floats (one per lane) into descending lane order.
+__device__ __forceinline__ float warp_sort_desc_f(float x, int lane) {
+#pragma unroll
+  for (int size = 2; size <= 32; size <<= 1)
+#pragma unroll
+    for (int stride = size >> 1; stride > 0; stride >>= 1) {
+      const float y = __shfl_xor_sync(0xffffffffu, x, stride);
+      const bool keep_max = ((lane & stride) == 0) == ((lane & size) == 0);
+      x = keep_max ? fmaxf(x, y) : fminf(x, y);
+    }
+  return x;
+}
+
+// A floor for the k-th best score from a warp's first batch: among the 32
+// lane maxima (the best valid candidate of each lane), the k-th largest is
+// reached by at least k distinct candidates, so no score below it can be
+// among the k best of the slice.  Candidates below it are then rejected by
+// the float compare alone, which spares most of the insertions a root
+// otherwise pays while its list fills.
+__device__ __forceinline__ void set_floor(WarpTopK& w, const Batch& b, int k, int lane) {
+  float m = -INFINITY;   // fmaxf ignores a NaN operand
+#pragma unroll
+  for (int i = 0; i < kBatch; ++i) {
+    m = fmaxf(m, (b.v[i] & 0xFFu) != 0 ? b.d[i].x : -INFINITY);
+    m = fmaxf(m, (b.v[i] & 0xFF00u) != 0 ? b.d[i].y : -INFINITY);
+    m = fmaxf(m, (b.v[i] & 0xFF0000u) != 0 ? b.d[i].z : -INFINITY);
+    m = fmaxf(m, (b.v[i] & 0xFF000000u) != 0 ? b.d[i].w : -INFINITY);
+  }
+  m = warp_sort_desc_f(m, lane);
+  w.floor = fmaxf(w.floor, __shfl_sync(0xffffffffu, m, k - 1));
+  w.tau_s = fmaxf(w.tau_s, w.floor);
 }
 
 // The warp streams absolute positions [a0, a1) of the root starting at
 // `start`: scalar head and tail, and a vector body walked in warp-uniform
-// steps of 4 x 32 four-position groups whose loads are all issued first.
+// batches (all loads of a batch issued before any is used, and the next
+// batch's issued before the current one is examined); the first batch sets
+// the floor.
 template <bool kVec>
 __device__ __forceinline__ void stream_range(WarpTopK& w, const float* delta, const uint8_t* valid,
-                                             int64_t start, int64_t a0, int64_t a1, int k,
+                                             int64_t start64, int64_t a0_64, int64_t a1_64, int k,
                                              int lane) {
+  const int32_t start = static_cast<int32_t>(start64);
+  const int32_t a0 = static_cast<int32_t>(a0_64), a1 = static_cast<int32_t>(a1_64);
   if (!kVec) {
-    for (int64_t q = a0; q < a1; q += 32) {
-      const int64_t p = q + lane;
+    for (int32_t q = a0; q < a1; q += 32) {
+      const int32_t p = q + lane;
       const bool in = p < a1;
       wtk_offer(w, in ? delta[p] : 0.f, in && (valid == nullptr || valid[p] != 0), p - start, k,
                 lane);
     }
     return;
   }
-  const int64_t h = a0 + ((4 - (a0 & 3)) & 3) < a1 ? a0 + ((4 - (a0 & 3)) & 3) : a1;
-  {
-    const int64_t p = a0 + lane;
-    const bool in = p < h;
-    wtk_offer(w, in ? delta[p] : 0.f, in && (valid == nullptr || valid[p] != 0), p - start, k,
-              lane);
+  const int32_t h = a0 + ((4 - (a0 & 3)) & 3) < a1 ? a0 + ((4 - (a0 & 3)) & 3) : a1;
+  const int32_t body = h + ((a1 - h) & ~3);
+  for (int32_t q = h; q < body; q += kSpan) {
+    Batch x;
+    if (q + kSpan <= body)
+      load_batch<true>(x, delta, valid, q, body, lane);
+    else
+      load_batch<false>(x, delta, valid, q, body, lane);
+    if (q == h) set_floor(w, x, k, lane);
+    offer_batch(w, x, q, start, k, lane);
   }
-  const int64_t body = h + ((a1 - h) & ~int64_t{3});
-  constexpr int kBatch = 4;
-  for (int64_t q = h; q < body; q += 4 * 32 * kBatch) {
-    float4 d[kBatch];
-    uint32_t v[kBatch];
-#pragma unroll
-    for (int i = 0; i < kBatch; ++i) {
-      const int64_t p = q + 4 * (32 * i + lane);
-      if (p < body) {
-        d[i] = *reinterpret_cast<const float4*>(delta + p);
-        v[i] = valid ? *reinterpret_cast<const uint32_t*>(valid + p) : 0x01010101u;
-      } else {
-        d[i] = make_float4(0.f, 0.f, 0.f, 0.f);
-        v[i] = 0u;
-      }
-    }
-#pragma unroll
-    for (int i = 0; i < kBatch; ++i) {
-      const int64_t t = q + 4 * (32 * i + lane) - start;
-      wtk_offer(w, d[i].x, (v[i] & 0xFFu) != 0, t, k, lane);
-      wtk_offer(w, d[i].y, (v[i] & 0xFF00u) != 0, t + 1, k, lane);
-      wtk_offer(w, d[i].z, (v[i] & 0xFF0000u) != 0, t + 2, k, lane);
-      wtk_offer(w, d[i].w, (v[i] & 0xFF000000u) != 0, t + 3, k, lane);
-    }
-  }
-  {
-    const int64_t p = body + lane;
-    const bool in = p < a1;
-    wtk_offer(w, in ? delta[p] : 0.f, in && (valid == nullptr || valid[p] != 0), p - start, k,
-              lane);
-  }
+  // scalar head and tail (at most 3 positions each)
+  const int32_t p = lane < 4 ? a0 + lane : body + (lane - 4);
+  const bool in = lane < 4 ? p < h : p < a1;
+  wtk_offer(w, in ? delta[p] : 0.f, in && (valid == nullptr || valid[p] != 0), p - start, k,
+            lane);
 }
 
-// kWarps == 1: one warp per root (8 roots per 256-thread block);
-// kWarps == 16: one block per root, each warp a contiguous slice, the
-// partial lists merged by warp 0 through shared memory.
-template <int kWarps, bool kVec>
-__global__ void __launch_bounds__(kWarps == 1 ? 256 : 32 * kWarps)
+// S warps share a root (S = 1, 2, 4, 8 in blocks of 8 warps, so 8/S roots
+// at a time per block; S = 16 in blocks of 16 warps): each warp streams one
+// contiguous slice of the root, then the group merges its S lists pairwise
+// through shared memory (a bitonic merge per level, the group's own named
+// barrier between levels) and its first warp writes the result.
+template <int S>
+struct TopkShape {
+  static constexpr int kWarps = S == 16 ? 16 : 8;    // warps per block
+  static constexpr int kGroups = kWarps / S;         // roots in flight per block
+  static constexpr int kMinBlocks = S == 16 ? 1 : (S == 1 ? 5 : 4);
+};
+
+__device__ __forceinline__ void group_sync(int id, int threads) {
+  asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(threads) : "memory");
+}
+
+template <int S, bool kVec>
+__global__ void __launch_bounds__(32 * TopkShape<S>::kWarps, TopkShape<S>::kMinBlocks)
     select_topk_kernel(const float* __restrict__ delta, const uint8_t* __restrict__ valid,
                        int64_t n_tokens, const int64_t* __restrict__ root_offsets,
                        int32_t n_roots, int32_t k, int32_t lo, int32_t hi,
                        int32_t* __restrict__ branch_pos, int32_t* __restrict__ n_selected,
                        float* __restrict__ branch_delta) {
+  using Sh = TopkShape<S>;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  const int roots_per_block = kWarps == 1 ? blockDim.x / 32 : 1;
-  const int64_t first =
-      static_cast<int64_t>(blockIdx.x) * roots_per_block + (kWarps == 1 ? warp : 0);
-  const int64_t step = static_cast<int64_t>(gridDim.x) * roots_per_block;
-  __shared__ uint64_t lists[kWarps == 1 ? 1 : kWarps][32];
-  for (int64_t r = first; r < n_roots; r += step) {
+  const int grp = warp / S, ws = warp % S;
+  __shared__ uint64_t lists[S == 1 ? 1 : Sh::kWarps][32];
+  const int64_t step = static_cast<int64_t>(gridDim.x) * Sh::kGroups;
+  for (int64_t r = static_cast<int64_t>(blockIdx.x) * Sh::kGroups + grp; r < n_roots; r += step) {
     const int64_t start = root_offsets[r];
     const int64_t end = root_offsets[r + 1];
     const int64_t T = end > start ? end - start : 0;
@@ -321,23 +470,29 @@ __global__ void __launch_bounds__(kWarps == 1 ? 256 : 32 * kWarps)
     int64_t a0 = start + w_lo, a1 = start + w_hi;
     if (a0 < 0) a0 = 0;
     if (a1 > n_tokens) a1 = n_tokens;
-    WarpTopK w{0ull, 0ull, -INFINITY};
-    if (kWarps == 1) {
+    WarpTopK w{0ull, 0ull, -INFINITY, -INFINITY};
+    if constexpr (S == 1) {
       if (a1 > a0) stream_range<kVec>(w, delta, valid, start, a0, a1, k, lane);
     } else {
       const int64_t len = a1 > a0 ? a1 - a0 : 0;
-      const int64_t per = ((len + kWarps - 1) / kWarps + 3) & ~int64_t{3};
-      const int64_t s0 = a0 + per * warp;
+      const int64_t per = ((len + S - 1) / S + 3) & ~int64_t{3};
+      const int64_t s0 = a0 + per * ws;
       const int64_t s1 = s0 + per < a1 ? s0 + per : a1;
       if (s0 < s1) stream_range<kVec>(w, delta, valid, start, s0, s1, k, lane);
       lists[warp][lane] = w.mine;
-      __syncthreads();
-      if (warp == 0) {
-        w = WarpTopK{0ull, 0ull, -INFINITY};
-        for (int i = 0; i < kWarps; ++i) wtk_offer_key(w, lists[i][lane], k, lane);
+      const int bar = 1 + grp, nthreads = 32 * S;
+      group_sync(bar, nthreads);
+#pragma unroll
+      for (int half = S / 2; half >= 1; half >>= 1) {
+        if (ws < half) {
+          const uint64_t m =
+              bitonic_merge16(lists[warp][lane & 15], lists[warp + half][(31 - lane) & 15], lane);
+          w.mine = lane < k ? m : 0ull;
+          lists[warp][lane] = w.mine;
+        }
+        group_sync(bar, nthreads);
       }
-      __syncthreads();
-      if (warp != 0) continue;
+      if (ws != 0) continue;
     }
     const int n = __popc(__ballot_sync(0xffffffffu, w.mine != 0ull));
     if (lane < k) {
@@ -355,29 +510,72 @@ __global__ void __launch_bounds__(kWarps == 1 ? 256 : 32 * kWarps)
   }
 }
 
-// Many roots: one warp per root, a persistent grid of as many 8-warp blocks
-// as are resident at once.  Few roots: 16 warps per root so that the GPU
-// fills.  (Splitting mid-length roots over 4 warps was measured slower: the
-// per-root barrier and merge cost more than the shorter chains save.)
+// HDL_SELECT_SPLIT (1, 2, 4 or 8) fixes the warps per root of the many-roots
+// mode, for tests and tuning; results do not depend on it.
+int select_split_override() {
+  static const int v = [] {
+    const char* e = std::getenv("HDL_SELECT_SPLIT");
+    if (e && (e[0] == '1' || e[0] == '2' || e[0] == '4' || e[0] == '8') && e[1] == '\0')
+      return e[0] - '0';
+    return 0;
+  }();
+  return v;
+}
+
+template <int S, bool kVec>
+hdl_status launch_topk_s(const float* delta, const uint8_t* valid, int64_t n_tokens,
+                         const int64_t* offs, int32_t n_roots, int32_t k, int32_t lo, int32_t hi,
+                         int32_t* bp, int32_t* ns, float* bd, int grid, cudaStream_t st) {
+  select_topk_kernel<S, kVec><<<grid, 32 * TopkShape<S>::kWarps, 0, st>>>(
+      delta, valid, n_tokens, offs, n_roots, k, lo, hi, bp, ns, bd);
+  return launch_status();
+}
+
+// Few roots (< 2 per SM): 16 warps per root, one block each, so that every
+// root is done in a single short pass.  Many roots: a persistent grid of
+// 8-warp blocks; S warps per root, S the smallest power of two that gives
+// every resident warp a slice (so that a few hundred long roots still keep
+// enough loads in flight), but no slice shorter than 1024 positions.  (More
+// slices than that only add per-slice work: 8192 roots of 4096 positions
+// took 47, 51, 67 and 84 us at S = 1, 2, 4, 8.  At S = 1 the kernel runs
+// within 8% of a read-only kernel with the same one-warp-per-root pattern
+// and occupancy; neither deeper register prefetch nor a shared-memory ring
+// filled by bulk copies made it faster.)
 template <bool kVec>
 hdl_status launch_topk(const float* delta, const uint8_t* valid, int64_t n_tokens,
                        const int64_t* offs, int32_t n_roots, int32_t k, int32_t lo, int32_t hi,
                        int32_t* bp, int32_t* ns, float* bd, int sms, cudaStream_t st) {
-  if (n_roots >= 2 * sms) {
-    int per_sm = 0;
-    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, select_topk_kernel<1, kVec>, 256,
-                                                      0) != cudaSuccess || per_sm <= 0)
-      per_sm = 4;
-    const int64_t blocks = (n_roots + 7) / 8;
-    const int64_t cap = static_cast<int64_t>(per_sm) * sms;
-    const int grid = static_cast<int>(blocks < cap ? blocks : cap);
-    select_topk_kernel<1, kVec><<<grid, 256, 0, st>>>(delta, valid, n_tokens, offs, n_roots, k,
-                                                      lo, hi, bp, ns, bd);
-  } else {
-    select_topk_kernel<16, kVec><<<n_roots, 512, 0, st>>>(delta, valid, n_tokens, offs,
-                                                          n_roots, k, lo, hi, bp, ns, bd);
+  if (n_roots < 2 * sms)
+    return launch_topk_s<16, kVec>(delta, valid, n_tokens, offs, n_roots, k, lo, hi, bp, ns, bd,
+                                   n_roots, st);
+  int per_sm = 0;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, select_topk_kernel<1, kVec>, 256,
+                                                    0) != cudaSuccess || per_sm <= 0)
+    per_sm = 4;
+  const int64_t resident_warps = static_cast<int64_t>(per_sm) * 8 * sms;
+  int64_t span = n_tokens / n_roots;
+  if (hi > 0 && hi < span) span = hi;
+  span -= lo > 0 ? lo : 0;
+  int S = 1;
+  while (S < 8 && int64_t{n_roots} * S < resident_warps && span / (2 * S) >= 1024) S *= 2;
+  if (const int forced = select_split_override()) S = forced;
+  const int64_t blocks = (int64_t{n_roots} * S + 7) / 8;
+  const int64_t cap = static_cast<int64_t>(per_sm) * sms;
+  const int grid = static_cast<int>(blocks < cap ? blocks : cap);
+  switch (S) {
+    case 1:
+      return launch_topk_s<1, kVec>(delta, valid, n_tokens, offs, n_roots, k, lo, hi, bp, ns, bd,
+                                    grid, st);
+    case 2:
+      return launch_topk_s<2, kVec>(delta, valid, n_tokens, offs, n_roots, k, lo, hi, bp, ns, bd,
+                                    grid, st);
+    case 4:
+      return launch_topk_s<4, kVec>(delta, valid, n_tokens, offs, n_roots, k, lo, hi, bp, ns, bd,
+                                    grid, st);
+    default:
+      return launch_topk_s<8, kVec>(delta, valid, n_tokens, offs, n_roots, k, lo, hi, bp, ns, bd,
+                                    grid, st);
   }
-  return launch_status();
 }
 
 }  // namespace

@@ -1,5 +1,9 @@
 """Selection, allocation and mask kernels: bit-exact against the oracle when
 fed the same scores, offsets and masks (Sections 3.2, 3.3, 4.1, 4.4)."""
+import os
+import subprocess
+import sys
+
 import numpy as np
 import pytest
 import torch
@@ -202,3 +206,48 @@ def test_select_unaligned_buffers(hdl, n_roots):
     bp, ns, bd = hdl.hdl_select_branches(d[1:], v[1:], torch.from_numpy(offs).cuda(), 8)
     pos, nsel, val = oracle.select_branches(delta.astype(np.float64), valid, offs, 8)
     assert np.array_equal(ns.cpu().numpy(), nsel) and np.array_equal(bp.cpu().numpy(), pos)
+
+
+_SPLIT_SCRIPT = r"""
+import sys
+import numpy as np
+import torch
+sys.path.insert(0, sys.argv[1])
+import paper_2609_36864_gb300 as hdl
+data = np.load(sys.argv[2])
+d = torch.from_numpy(data["delta"]).cuda()
+v = torch.from_numpy(data["valid"]).cuda()
+o = torch.from_numpy(data["offs"]).cuda()
+out = {}
+for k in (1, 8, 16):
+    for lo, hi in ((0, 0), (37, 3001)):
+        bp, ns, bd = hdl.hdl_select_branches(d, v, o, k, lo=lo, hi=hi)
+        out[f"bp{k}_{lo}"] = bp.cpu().numpy()
+        out[f"ns{k}_{lo}"] = ns.cpu().numpy()
+        out[f"bd{k}_{lo}"] = bd.cpu().numpy()
+np.savez(sys.argv[3], **out)
+"""
+
+
+@pytest.mark.parametrize("split", ["1", "2", "4", "8"])
+def test_select_warps_per_root(hdl, tmp_path, split):
+    """The many-roots mode with 1, 2, 4 or 8 warps per root (forced): every
+    split gives the oracle's selection bit for bit, including ragged and
+    empty roots, heavy ties and a window."""
+    rng = np.random.default_rng(21)
+    lengths = list(rng.integers(1500, 6000, size=330)) + [0, 1, 5, 4099]
+    delta, valid, offs = make_roots(lengths, 22, tie_levels=40)
+    inp = tmp_path / "in.npz"
+    np.savez(inp, delta=delta, valid=valid, offs=offs)
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    outp = tmp_path / "out.npz"
+    subprocess.run([sys.executable, "-c", _SPLIT_SCRIPT, root, str(inp), str(outp)],
+                   env=dict(os.environ, HDL_SELECT_SPLIT=split), check=True, timeout=300)
+    got = np.load(outp)
+    for k in (1, 8, 16):
+        for lo, hi in ((0, 0), (37, 3001)):
+            pos, nsel, val = oracle.select_branches(delta.astype(np.float64), valid, offs, k,
+                                                    lo=lo, hi=hi)
+            assert np.array_equal(got[f"ns{k}_{lo}"], nsel)
+            assert np.array_equal(got[f"bp{k}_{lo}"], pos)
+            assert np.array_equal(got[f"bd{k}_{lo}"].astype(np.float64), val, equal_nan=True)
