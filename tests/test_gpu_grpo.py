@@ -18,6 +18,18 @@ def hdl():
     return m
 
 
+def decided(lpn, lpo, eps_low=0.2, eps_high=0.28):
+    """Tokens whose clip decision both sides must take alike: the float32
+    ratio is more than 2 ulp from 1 - eps_low and 1 + eps_high (CUDA's expf
+    and numpy's float32 exp may round differently by up to 2 ulp, which can
+    flip the decision right at a bound)."""
+    r = np.exp(lpn.astype(np.float32) - lpo.astype(np.float32)).astype(np.float64)
+    ok = np.ones(len(r), dtype=bool)
+    for b in (np.float32(1.0) - np.float32(eps_low), np.float32(1.0) + np.float32(eps_high)):
+        ok &= np.abs(r - float(b)) > 2 * float(np.spacing(b))
+    return ok
+
+
 def make_batch(seed, n_groups, max_len):
     rng = np.random.default_rng(seed)
     sizes = rng.integers(1, 17, size=n_groups)
@@ -35,7 +47,10 @@ def make_batch(seed, n_groups, max_len):
     return lpn, lpo, mask, toffs, rewards, goffs
 
 
-@pytest.mark.parametrize("seed,n_groups,max_len", [(0, 40, 300), (1, 8, 5000), (2, 300, 30)])
+# (3, 20000, 21): ~170K short (and empty) trajectories, so that a warp's
+# share of the tokens spans more than 31 of them
+@pytest.mark.parametrize("seed,n_groups,max_len", [(0, 40, 300), (1, 8, 5000), (2, 300, 30),
+                                                   (3, 20000, 21)])
 def test_grpo_loss_matches_oracle(hdl, seed, n_groups, max_len):
     lpn, lpo, mask, toffs, R, goffs = make_batch(seed, n_groups, max_len)
     t = lambda x: torch.from_numpy(x).cuda()
@@ -52,8 +67,9 @@ def test_grpo_loss_matches_oracle(hdl, seed, n_groups, max_len):
     assert abs(st[2] - clip_frac) <= 1e-6
     assert abs(st[3] - mean_r) <= 1e-5
     g = grad.cpu().numpy()
-    assert np.all((g == 0) == (g_ref == 0))
-    assert np.all(np.abs(g - g_ref) <= 1e-5 * np.abs(g_ref).max())
+    ok = decided(lpn, lpo)
+    assert np.all((g == 0)[ok] == (g_ref == 0)[ok])
+    assert np.all(np.abs(g - g_ref)[ok] <= 1e-5 * np.abs(g_ref).max())
     assert np.all(g[mask == 0] == 0)
 
 
@@ -93,4 +109,5 @@ def test_grpo_unaligned(hdl, shift):
     assert st[1] == n and abs(st[0] - loss) <= 1e-5 * max(1.0, abs(loss))
     g = grad.cpu().numpy()
     assert np.all(g[:shift] == 0)
-    assert np.all(np.abs(g[shift:] - g_ref) <= 1e-5 * np.abs(g_ref).max())
+    ok = decided(lpn, lpo)
+    assert np.all(np.abs(g[shift:] - g_ref)[ok] <= 1e-5 * np.abs(g_ref).max())
