@@ -49,6 +49,8 @@ def parse():
                         "(for launch-bound workloads such as tiny)")
     p.add_argument("--no-cpu", action="store_true")
     p.add_argument("--cpu-seconds", type=float, default=12.0)
+    p.add_argument("--digest", nargs="+", default=None, metavar="FILE",
+                   help="print the comment-insensitive digest of csrc/FILE... and exit")
     p.add_argument("--micro", default=None, choices=["select", "mask", "grpo"],
                    help="bandwidth micro-benchmark of one HBM-bound kernel at a scaled size")
     return p.parse_args()
@@ -72,14 +74,15 @@ def peaks():
     return 1900.0, 1700.0, 6800.0, "fallback"
 
 
-def kernel_source_digest() -> str:
-    """sha256 (16 hex digits) of the re-scoring kernel's sources with comments
-    and whitespace removed: what a DRAM-traffic record was measured on."""
+def kernel_source_digest(files=("rescore.cu", "ptx_sm103.cuh")) -> str:
+    """sha256 (16 hex digits) of kernel sources (default: the re-scoring
+    kernel's) with comments and whitespace removed: what a profile record was
+    measured on.  `python bench.py --digest select.cu` prints one."""
     import hashlib
     import re
     csrc = os.path.join(ROOT, "paper_2609_36864_gb300", "csrc")
     h = hashlib.sha256()
-    for f in ("rescore.cu", "ptx_sm103.cuh"):
+    for f in files:
         text = open(os.path.join(csrc, f)).read()
         text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
         text = re.sub(r"//[^\n]*", "", text)
@@ -539,6 +542,9 @@ def run_micro(args):
 
 def main():
     args = parse()
+    if args.digest:
+        print(kernel_source_digest(tuple(args.digest)))
+        return
     if args.micro:
         run_micro(args)
         return

@@ -190,7 +190,7 @@ __global__ void __launch_bounds__(kThreads, 4)
   int ntok = 0;
   // tokens [s, e) of one trajectory, advantage A: head and tail one token
   // per lane, the 16-byte-aligned body two 4-token groups per lane at a time
-  auto piece = [&](int64_t s, int64_t e, float A) {
+  auto stream_trajectory = [&](int64_t s, int64_t e, float A) {
     auto one = [&](int64_t u) {
       float g = 0.f;
       if (mask[u] != 0) {
@@ -249,7 +249,7 @@ __global__ void __launch_bounds__(kThreads, 4)
     int64_t ts = traj_offsets[j], te = traj_offsets[j + 1];
     ts = ts < 0 ? 0 : ts;
     te = te > n_tokens ? n_tokens : te;
-    if (te > ts) piece(ts, te, adv[j]);
+    if (te > ts) stream_trajectory(ts, te, adv[j]);
   }
   const float s0 = block_sum_f(acc.obj, red);
   const float s1 = block_sum_f(static_cast<float>(ntok), red);

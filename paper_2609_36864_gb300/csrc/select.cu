@@ -396,10 +396,9 @@ __device__ __forceinline__ void set_floor(WarpTopK& w, const Batch& b, int k, in
 }
 
 // The warp streams absolute positions [a0, a1) of the root starting at
-// `start`: scalar head and tail, and a vector body walked in warp-uniform
-// batches (all loads of a batch issued before any is used, and the next
-// batch's issued before the current one is examined); the first batch sets
-// the floor.
+// `start`: a vector body walked in warp-uniform batches (all loads of a
+// batch issued before any is used; the first batch sets the floor), then the
+// scalar head and tail.
 template <bool kVec>
 __device__ __forceinline__ void stream_range(WarpTopK& w, const float* delta, const uint8_t* valid,
                                              int64_t start64, int64_t a0_64, int64_t a1_64, int k,
