@@ -251,3 +251,34 @@ def test_select_warps_per_root(hdl, tmp_path, split):
             assert np.array_equal(got[f"ns{k}_{lo}"], nsel)
             assert np.array_equal(got[f"bp{k}_{lo}"], pos)
             assert np.array_equal(got[f"bd{k}_{lo}"].astype(np.float64), val, equal_nan=True)
+
+
+def test_select_randomized(hdl):
+    """40 seeded random configurations around the launch-mode boundaries
+    (2 roots per SM; few long roots, where the heuristic splits a root over
+    several warps; many short ones), with windows, ties, NaNs, invalid runs
+    and every k: bit-exact against the oracle."""
+    rng = np.random.default_rng(2024)
+    sms = torch.cuda.get_device_properties(0).multi_processor_count
+    for case in range(40):
+        kind = case % 4
+        if kind == 0:
+            R = int(rng.integers(2 * sms - 3, 2 * sms + 4))
+            lengths = rng.integers(0, 3000, size=R)
+        elif kind == 1:
+            R = int(rng.integers(2 * sms, 2 * sms + 200))
+            lengths = rng.integers(8000, 20000, size=R)
+        elif kind == 2:
+            R = int(rng.integers(1, 40))
+            lengths = rng.integers(0, 20000, size=R)
+        else:
+            R = int(rng.integers(1000, 3000))
+            lengths = rng.integers(0, 400, size=R)
+        ties = [None, 2, 50][case % 3]
+        delta, valid, offs = make_roots(list(lengths), 100 + case, tie_levels=ties,
+                                        nan_frac=0.01 * (case % 2),
+                                        invalid_frac=float(rng.choice([0.0, 0.2, 0.9])))
+        k = int(rng.integers(1, 17))
+        lo, hi = [(0, 0), (int(rng.integers(0, 500)), 0), (0, int(rng.integers(1, 9000))),
+                  (int(rng.integers(0, 300)), int(rng.integers(300, 12000)))][case % 4]
+        assert_select_equal(hdl, delta, valid if case % 5 else None, offs, k, lo=lo, hi=hi)
