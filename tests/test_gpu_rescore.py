@@ -177,3 +177,30 @@ def test_rescore_entropy(hdl, n, d, V, dt):
     assert_logp_close(e1.cpu().numpy(), oracle.next_token_entropy(h1, W), "entropy hind")
     if V == 1:
         assert torch.all(e0.abs() < 1e-6)
+
+
+def _tf32(x: np.ndarray, nearest: bool) -> np.ndarray:
+    """fp32 -> tf32 (10 mantissa bits) as fp64: round to nearest even, or truncate."""
+    b = np.ascontiguousarray(x, dtype=np.float32).view(np.uint32).astype(np.uint64)
+    if nearest:
+        b = b + 0xFFF + ((b >> 13) & 1)
+    b = (b & 0xFFFFE000) & 0xFFFFFFFF
+    return b.astype(np.uint32).view(np.float32).astype(np.float64)
+
+
+def test_rescore_tf32_rounds_to_nearest(hdl):
+    """fp32 inputs are rounded to tf32 to nearest (as the header states): the
+    kernel matches the oracle on round-to-nearest tf32 inputs at fp32
+    accumulation precision, and a truncating rounding is far from it."""
+    spec = hdl_synth.small_spec("tf32rn", n_roots=1, t_lo=300, t_hi=300, d=512, vocab=3000,
+                                dtype="f32", seed=77)
+    wl = hdl_synth.generate(spec, device="cuda")
+    lp0, lp1, _, ws = hdl.hdl_rescore(wl.h_orig, wl.h_hind, wl.w, wl.targets)
+    assert hdl.hdl_device_status(ws)[0] == hdl.HDL_OK
+    got = lp0.cpu().numpy().astype(np.float64)
+    h, w = wl.h_orig.cpu().numpy(), wl.w.cpu().numpy()
+    y = wl.targets.cpu().numpy()
+    err_rn = np.abs(got - oracle_logprobs(_tf32(h, True), _tf32(w, True), y)).max()
+    err_tr = np.abs(got - oracle_logprobs(_tf32(h, False), _tf32(w, False), y)).max()
+    assert err_rn < 5e-5, err_rn
+    assert err_tr > 4 * err_rn, (err_tr, err_rn)
