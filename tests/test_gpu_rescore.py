@@ -204,3 +204,37 @@ def test_rescore_tf32_rounds_to_nearest(hdl):
     err_tr = np.abs(got - oracle_logprobs(_tf32(h, False), _tf32(w, False), y)).max()
     assert err_rn < 5e-5, err_rn
     assert err_tr > 4 * err_rn, (err_tr, err_rn)
+
+
+@pytest.mark.parametrize("V", [1, 257, 4096, 32000])
+def test_rescore_zero_states_give_uniform(hdl, V):
+    """All-zero hidden states: every logit is 0, so log p = -ln V for every
+    token in both contexts and Delta = 0 (the closed form of a uniform
+    distribution; V = 1 gives 0)."""
+    n, d = 333, 128
+    h = torch.zeros((n, d), dtype=torch.bfloat16, device="cuda")
+    w = (torch.randn((V, d), device="cuda") * 0.02).to(torch.bfloat16)
+    y = torch.randint(0, V, (n,), dtype=torch.int32, device="cuda")
+    lp0, lp1, de, ws = hdl.hdl_rescore(h, h.clone(), w, y)
+    assert hdl.hdl_device_status(ws)[0] == hdl.HDL_OK
+    ref = -np.log(V)
+    assert np.all(np.abs(lp0.cpu().numpy() - ref) <= 1e-5 * max(1.0, abs(ref)))
+    assert torch.equal(lp0, lp1) and torch.all(de == 0)
+
+
+def test_rescore_large_logits(hdl):
+    """Hidden states scaled 64x (logits in the hundreds, log-probs down to
+    -10^3): the online max/sum stays finite and matches the oracle."""
+    spec = hdl_synth.small_spec("big", n_roots=1, t_lo=400, t_hi=400, d=256, vocab=5000,
+                                dtype="bf16", seed=91)
+    wl = hdl_synth.generate(spec, device="cuda")
+    h0 = (wl.h_orig.float() * 64).to(torch.bfloat16)
+    h1 = (wl.h_hind.float() * 64).to(torch.bfloat16)
+    lp0, lp1, de, ws = hdl.hdl_rescore(h0, h1, wl.w, wl.targets)
+    assert hdl.hdl_device_status(ws)[0] == hdl.HDL_OK
+    W = to_f64(wl.w)
+    y = wl.targets.cpu().numpy()
+    r0 = oracle_logprobs(to_f64(h0), W, y)
+    assert np.isfinite(lp0.cpu().numpy()).all() and r0.min() < -50
+    assert_logp_close(lp0.cpu().numpy(), r0, "large orig")
+    assert_logp_close(lp1.cpu().numpy(), oracle_logprobs(to_f64(h1), W, y), "large hind")
