@@ -198,8 +198,8 @@ HDL_API hdl_status hdl_merge_vocab_shards(const float* stats, int32_t n_shards,
  *   group_offsets   [n_groups + 1] int32: group g = trajectories
  *                   [group_offsets[g], group_offsets[g+1]).
  *   eps_low, eps_high  clip thresholds, 0 <= eps_low < 1, eps_high >= 0.
- *   advantages      [n_traj] float out (trajectories outside every group are
- *                   not written).
+ *   advantages      [n_traj] float out, NULL only when n_traj == 0
+ *                   (trajectories outside every group are not written).
  *   grad            [n_tokens] float out or NULL.
  *   stats           [4] float out: loss, masked tokens, fraction of masked
  *                   tokens whose clipped term is strictly smaller, mean ratio.

@@ -306,12 +306,12 @@ extern "C" hdl_status hdl_grpo_loss(const float* logp_new, const float* logp_old
                                     void* cuda_stream) {
   if (n_tokens < 0 || n_traj < 0 || n_groups < 0) return HDL_ERR_INVALID_ARG;
   if (!(eps_low >= 0.f && eps_low < 1.f && eps_high >= 0.f)) return HDL_ERR_INVALID_ARG;
-  if (!stats || !advantages || (n_groups > 0 && (!rewards || !group_offsets)))
+  if (!stats || (n_traj > 0 && !advantages) || (n_groups > 0 && (!rewards || !group_offsets)))
     return HDL_ERR_INVALID_ARG;
   if (n_traj > 0 && !traj_offsets) return HDL_ERR_INVALID_ARG;
   if (n_tokens > 0 && (!logp_new || !logp_old || !mask || n_traj == 0))
     return HDL_ERR_INVALID_ARG;
-  if (!aligned_to(stats, 4) || !aligned_to(advantages, 4) ||
+  if (!aligned_to(stats, 4) || (advantages && !aligned_to(advantages, 4)) ||
       (traj_offsets && !aligned_to(traj_offsets, 8)) ||
       (group_offsets && !aligned_to(group_offsets, 4)) || (grad && !aligned_to(grad, 4)))
     return HDL_ERR_INVALID_ARG;

@@ -111,3 +111,20 @@ def test_grpo_unaligned(hdl, shift):
     assert np.all(g[:shift] == 0)
     ok = decided(lpn, lpo)
     assert np.all(np.abs(g[shift:] - g_ref)[ok] <= 1e-5 * np.abs(g_ref).max())
+
+
+def test_grpo_empty_inputs(hdl):
+    """No tokens and no trajectories: the call succeeds and every statistic is
+    0.  Groups but no tokens: the advantages are still R - group mean."""
+    e32 = torch.empty(0, dtype=torch.float32, device="cuda")
+    eu8 = torch.empty(0, dtype=torch.uint8, device="cuda")
+    zero64 = torch.zeros(1, dtype=torch.int64, device="cuda")
+    zero32 = torch.zeros(1, dtype=torch.int32, device="cuda")
+    adv, grad, stats = hdl.hdl_grpo_loss(e32, e32, eu8, zero64, e32, zero32)
+    assert adv.numel() == 0 and torch.all(stats == 0)
+    R = np.array([0.25, 1.0, 0.5], dtype=np.float32)
+    adv, grad, stats = hdl.hdl_grpo_loss(
+        e32, e32, eu8, torch.zeros(4, dtype=torch.int64, device="cuda"),
+        torch.from_numpy(R).cuda(), torch.tensor([0, 3], dtype=torch.int32, device="cuda"))
+    assert np.allclose(adv.cpu().numpy(), R - R.astype(np.float64).mean(), rtol=0, atol=1e-7)
+    assert torch.all(stats == 0)
