@@ -282,3 +282,22 @@ def test_select_randomized(hdl):
         lo, hi = [(0, 0), (int(rng.integers(0, 500)), 0), (0, int(rng.integers(1, 9000))),
                   (int(rng.integers(0, 300)), int(rng.integers(300, 12000)))][case % 4]
         assert_select_equal(hdl, delta, valid if case % 5 else None, offs, k, lo=lo, hi=hi)
+
+
+def test_empty_inputs_through_the_binding(hdl):
+    """Zero roots; roots that are all empty (no tokens at all); zero
+    continuations: every call succeeds and writes what the empty case means."""
+    e32 = torch.empty(0, dtype=torch.float32, device="cuda")
+    eu8 = torch.empty(0, dtype=torch.uint8, device="cuda")
+    bp, ns, bd = hdl.hdl_select_branches(e32, eu8, torch.zeros(1, dtype=torch.int64,
+                                                                device="cuda"), 4)
+    assert bp.numel() == 0 and ns.numel() == 0
+    offs = torch.zeros(6, dtype=torch.int64, device="cuda")          # 5 empty roots
+    bp, ns, bd = hdl.hdl_select_branches(e32, eu8, offs, 4)
+    assert torch.all(ns == 0) and torch.all(bp == -1) and torch.all(torch.isnan(bd))
+    conts = torch.zeros(5, dtype=torch.int32, device="cuda")
+    cb = hdl.hdl_assign_continuations(ns, bp, conts, n_cont=0)
+    assert cb.numel() == 0
+    m = hdl.hdl_suffix_mask(cb, torch.zeros(1, dtype=torch.int64, device="cuda"), None,
+                            mask_len=0)
+    assert m.numel() == 0
