@@ -9,7 +9,7 @@ What is modelled (Section 3 of the paper): one problem's root trajectories
 y = (y_1..y_T), the final-layer hidden state of every root token under the
 original context (x, y_<i) and under the hindsight context (x, h, y_<i) of
 Eq. (hindsight-contexts), the LM-head matrix W shared by both contexts, the
-"policy-generated token" mask (agent trajectories interleave environment
+mask of tokens the policy generated itself (agent trajectories interleave environment
 observations, Section 4.1 "Tasks"), and the continuation layout of Section 3.3
 (each continuation reuses its root's prefix and, in this stand-in, has the
 root's length and validity pattern).

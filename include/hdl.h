@@ -264,7 +264,8 @@ HDL_API hdl_status hdl_device_status(const void* workspace, size_t workspace_byt
 /* ------------------------------------------------------------------------
  * Branch-point selection (Section 3.2: rank each root's candidate positions
  * by delta and take the highest; Section 3.1: only policy-generated tokens
- * are candidates; Section 4.4: points "too close together" keep only one).
+ * are candidates; Section 4.4: of points that sit too near each other only
+ * one is kept).
  *
  * For root r the candidates are positions t (relative to the root start) in
  * the window [lo, hi) -- hi <= 0 means the root's end -- with valid != 0 and

@@ -17,8 +17,8 @@ Functions and the passages they follow (arXiv 2609.36864):
   select_branches        Section 3.2 (rank the candidate positions of a root by
                          s_i, take the highest), candidates = policy-generated
                          tokens (Section 3.1); optional spacing rule of
-                         Section 4.4 ("points too close together: only one is
-                         retained").
+                         Section 4.4 (of points that sit too near each other,
+                         one is kept).
   allocate_counts        Section 4.1 "Rollout protocols" (2 points, 3 + 4
                          continuations, G = 2 x (1 + 3 + 4) = 16), Table
                          (fork-ablation) 2x1 -> 7 and 4x2 -> 1 + 2, and
@@ -37,7 +37,7 @@ Readings where the paper is silent (each is also listed in the design notes):
   * ties in s_i go to the lower position;
   * fewer than k candidates: all of them are returned, the rest padded with -1;
   * NaN scores are not candidates;
-  * the spacing rule takes min_gap (|t - a| < min_gap is "too close") with two
+  * the spacing rule takes min_gap (|t - a| < min_gap counts as too close) with two
     modes: greedy (walk the ranked list, skip a point too close to an accepted
     one) and drop-lower (take the plain top k, then drop each point too close
     to an accepted higher-ranked one);
