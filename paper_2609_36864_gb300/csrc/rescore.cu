@@ -602,12 +602,34 @@ PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
   return fn;
 }
 
+// The driver's tensor-map encoder needs a context current in the calling
+// thread.  A host thread whose first CUDA call is into this library has none
+// yet (the library's runtime is linked statically and binds contexts lazily,
+// on its first call that needs one), so bind the current device's primary
+// context first -- unless the thread already has a context current.
+bool ensure_context() {
+  static PFN_cuCtxGetCurrent_v4000 get_current = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 4000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      get_current = reinterpret_cast<PFN_cuCtxGetCurrent_v4000>(p);
+  });
+  CUcontext c = nullptr;
+  if (get_current && get_current(&c) == CUDA_SUCCESS && c != nullptr) return true;
+  int dev = 0;
+  return cudaGetDevice(&dev) == cudaSuccess && cudaSetDevice(dev) == cudaSuccess;
+}
+
 // 2-D row-major [rows, d] operand, boxes of (128 bytes of K) x box_rows,
 // 128-byte swizzle; rows past the end read as zeros.
 bool make_operand_map(CUtensorMap* m, const void* ptr, int64_t rows, int32_t d, int esize,
                       int box_rows) {
   auto enc = tensor_map_encoder();
-  if (!enc) return false;
+  if (!enc || !ensure_context()) return false;
   cuuint64_t dims[2] = {static_cast<cuuint64_t>(d), static_cast<cuuint64_t>(rows)};
   cuuint64_t strides[1] = {static_cast<cuuint64_t>(d) * esize};
   cuuint32_t box[2] = {static_cast<cuuint32_t>(kRowBytes / esize),

@@ -238,3 +238,47 @@ def test_rescore_large_logits(hdl):
     assert np.isfinite(lp0.cpu().numpy()).all() and r0.min() < -50
     assert_logp_close(lp0.cpu().numpy(), r0, "large orig")
     assert_logp_close(lp1.cpu().numpy(), oracle_logprobs(to_f64(h1), W, y), "large hind")
+
+
+def test_rescore_concurrent_host_threads(hdl):
+    """Two host threads, each on its own stream and workspace, calling the
+    library at the same time: every result is bit-identical to the same call
+    made alone (the library keeps no per-call state)."""
+    import threading
+    wls = [hdl_synth.generate(hdl_synth.small_spec(f"thr{i}", n_roots=2, t_lo=300, t_hi=500,
+                                                   d=256, vocab=5000, seed=300 + i),
+                              device="cuda") for i in range(2)]
+    ref = []
+    for wl in wls:
+        lp0, lp1, de, _ = hdl.hdl_rescore(wl.h_orig, wl.h_hind, wl.w, wl.targets)
+        bp, ns, bd = hdl.hdl_select_branches(de, wl.valid, wl.root_offsets, 8)
+        ref.append((lp0, lp1, de, bp, ns))
+    torch.cuda.synchronize()
+    out = [None, None]
+    errors = []
+
+    def work(i):
+        try:
+            s = torch.cuda.Stream()
+            wl = wls[i]
+            res = []
+            for _ in range(20):
+                lp0, lp1, de, _ = hdl.hdl_rescore(wl.h_orig, wl.h_hind, wl.w, wl.targets,
+                                                  stream=s)
+                bp, ns, bd = hdl.hdl_select_branches(de, wl.valid, wl.root_offsets, 8, stream=s)
+                res.append((lp0, lp1, de, bp, ns))
+            s.synchronize()
+            out[i] = res
+        except Exception as e:   # surfaced below
+            errors.append(e)
+
+    ts = [threading.Thread(target=work, args=(i,)) for i in range(2)]
+    for t in ts:
+        t.start()
+    for t in ts:
+        t.join()
+    assert not errors, errors
+    for i in range(2):
+        for res in out[i]:
+            for a, b in zip(res, ref[i]):
+                assert torch.equal(a, b)
