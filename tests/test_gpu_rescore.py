@@ -282,3 +282,18 @@ def test_rescore_concurrent_host_threads(hdl):
         for res in out[i]:
             for a, b in zip(res, ref[i]):
                 assert torch.equal(a, b)
+
+
+@pytest.mark.parametrize("d,dt", [(8192, "bf16"), (16384, "bf16"), (8192, "f32")])
+def test_rescore_wide_hidden(hdl, d, dt):
+    """Hidden sizes of 70B-class models and beyond (long K loops: up to 256
+    pipeline stages per tile) against the oracle."""
+    spec = hdl_synth.small_spec(f"wide{d}{dt}", n_roots=1, t_lo=200, t_hi=200, d=d, vocab=1500,
+                                dtype=dt, seed=d // 64)
+    wl = hdl_synth.generate(spec, device="cuda")
+    lp0, lp1, de, ws = hdl.hdl_rescore(wl.h_orig, wl.h_hind, wl.w, wl.targets)
+    assert hdl.hdl_device_status(ws)[0] == hdl.HDL_OK
+    W = to_f64(wl.w)
+    y = wl.targets.cpu().numpy()
+    assert_logp_close(lp0.cpu().numpy(), oracle_logprobs(to_f64(wl.h_orig), W, y), "wide orig")
+    assert_logp_close(lp1.cpu().numpy(), oracle_logprobs(to_f64(wl.h_hind), W, y), "wide hind")
