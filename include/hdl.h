@@ -191,7 +191,7 @@ HDL_API hdl_status hdl_merge_vocab_shards(const float* stats, int32_t n_shards,
  *   logp_new, logp_old  [n_tokens] float, packed trajectories.
  *   mask            [n_tokens] uint8: the loss mask (hdl_suffix_mask for
  *                   continuations, the valid mask for roots).
- *   traj_offsets    [n_traj + 1] int64: trajectory j = tokens
+ *   traj_offsets    [n_traj + 1] int64, non-decreasing: trajectory j = tokens
  *                   [traj_offsets[j], traj_offsets[j+1]); they should cover
  *                   [0, n_tokens) (tokens outside every trajectory carry no loss).
  *   rewards         [n_traj] float verifier rewards.

@@ -31,30 +31,26 @@ struct Sums {
   float obj, tokens, clipped, ratio;
 };
 
-__device__ __forceinline__ float block_sum_f(float v, float* red) {
+// Block-wide sums of four values per thread (warp shuffle trees, then
+// thread 0 adds the warps' sums in order); valid in thread 0.
+template <typename T>
+__device__ __forceinline__ void block_sum4(T (&v)[4], T (*red)[4]) {
 #pragma unroll
-  for (int o = 16; o >= 1; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  if (lane == 0) red[warp] = v;
-  __syncthreads();
-  float r = 0.f;
-  if (threadIdx.x == 0)
-    for (int w = 0; w < kThreads / 32; ++w) r += red[w];
-  __syncthreads();
-  return r;   // valid in thread 0
-}
-
-__device__ __forceinline__ double block_sum(double v, double* red) {
+  for (int i = 0; i < 4; ++i)
 #pragma unroll
-  for (int o = 16; o >= 1; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    for (int o = 16; o >= 1; o >>= 1) v[i] += __shfl_xor_sync(0xffffffffu, v[i], o);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  if (lane == 0) red[warp] = v;
+  if (lane == 0)
+#pragma unroll
+    for (int i = 0; i < 4; ++i) red[warp][i] = v[i];
   __syncthreads();
-  double r = 0.0;
-  if (threadIdx.x == 0)
-    for (int w = 0; w < kThreads / 32; ++w) r += red[w];
-  __syncthreads();
-  return r;   // valid in thread 0
+  if (threadIdx.x == 0) {
+#pragma unroll
+    for (int i = 0; i < 4; ++i) v[i] = red[0][i];
+    for (int w = 1; w < kThreads / 32; ++w)
+#pragma unroll
+      for (int i = 0; i < 4; ++i) v[i] += red[w][i];
+  }
 }
 
 // Bit 8i of the result is set iff byte i of w is nonzero.
@@ -152,11 +148,35 @@ __device__ __forceinline__ float token_grad(float lpn, float lpo, float A, float
   return active ? u * scale : 0.f;
 }
 
-// Token pass, one warp per trajectory (warps loop over trajectories): the
-// advantage is a warp-uniform scalar, the trajectory's tokens are streamed
-// with 16-byte loads, three 4-token groups per lane in flight (64 registers:
-// four more would cost occupancy; two measured 1 % slower).
-template <bool kVec>
+// The trajectory holding position a: the largest j < n with offs[j] <= a
+// (offsets non-decreasing, offs[0] <= a < offs[n]).  Each step the 32 lanes
+// probe 32 evenly spaced candidates and keep the last one not past a, so the
+// interval shrinks 32-fold per dependent load.
+__device__ __forceinline__ int64_t find_traj(const int64_t* __restrict__ offs, int32_t n,
+                                             int64_t a, int lane) {
+  int64_t lo_j = 0, hi_j = n - 1;
+  while (lo_j < hi_j) {
+    const int64_t step = (hi_j - lo_j + 32) / 32;
+    const int64_t c = lo_j + step * lane;
+    const bool ok = c <= hi_j && offs[c] <= a;
+    const unsigned m = __ballot_sync(0xffffffffu, ok);
+    const int top = m ? 31 - __clz(static_cast<int>(m)) : 0;
+    lo_j += step * top;
+    hi_j = lo_j + step - 1 < hi_j ? lo_j + step - 1 : hi_j;
+  }
+  return lo_j;
+}
+
+// Token pass.  Many trajectories (kFlat = false): one warp per trajectory
+// (warps loop over trajectories), its advantage a warp-uniform scalar.  Fewer
+// trajectories than about twice the resident warps (kFlat = true): warp w
+// takes the w-th of equal token ranges of [offs[0], offs[n]), finds the
+// trajectory holding its first token and walks the trajectories it overlaps
+// (their offsets and advantages read 32 at a time, one per lane), so a few
+// long trajectories still keep every warp streaming.  Either way the tokens
+// are streamed with 16-byte loads, three 4-token groups per lane in flight
+// (64 registers: four more would cost occupancy; two measured 1 % slower).
+template <bool kVec, bool kFlat>
 __global__ void __launch_bounds__(kThreads, 4)
     grpo_token_kernel(const float* __restrict__ lpn, const float* __restrict__ lpo,
                       const uint8_t* __restrict__ mask, int64_t n_tokens,
@@ -165,8 +185,8 @@ __global__ void __launch_bounds__(kThreads, 4)
                       const unsigned long long* __restrict__ counts, int n_count_blocks,
                       float* __restrict__ grad, Sums* __restrict__ partial,
                       unsigned int* __restrict__ done, float* __restrict__ stats) {
-  __shared__ float red[kThreads / 32];
-  __shared__ double red_d[kThreads / 32];
+  __shared__ float red[kThreads / 32][4];
+  __shared__ double red_d[kThreads / 32][4];
   __shared__ float s_scale;
   __shared__ bool s_last;
   if (threadIdx.x < 32) {   // the denominator: an exact integer sum, one warp
@@ -206,7 +226,7 @@ __global__ void __launch_bounds__(kThreads, 4)
       body = h + ((e - h) & ~int64_t{3});
     }
     if (lane < h - s) one(s + lane);
-    constexpr int kBatch = 3;
+    constexpr int kBatch = kFlat ? 2 : 3;   // the flat walk holds its window too
     for (int64_t q = h; q < body; q += 4 * 32 * kBatch) {
       float4 pn[kBatch], po[kBatch];
       uint32_t mv[kBatch];
@@ -240,43 +260,64 @@ __global__ void __launch_bounds__(kThreads, 4)
     }
     for (int64_t u = body + lane; u < e; u += 32) one(u);
   };
-  // one warp per trajectory (warps loop over trajectories).  (Equal token
-  // ranges per warp instead, each starting with a search for its first
-  // trajectory, measured slower: 167 against 158 us on 16384 x 4096.)
   const int64_t nw = static_cast<int64_t>(gridDim.x) * (kThreads / 32);
-  for (int64_t j = static_cast<int64_t>(blockIdx.x) * (kThreads / 32) + (threadIdx.x >> 5);
-       j < n_traj; j += nw) {
-    int64_t ts = traj_offsets[j], te = traj_offsets[j + 1];
-    ts = ts < 0 ? 0 : ts;
-    te = te > n_tokens ? n_tokens : te;
-    if (te > ts) stream_trajectory(ts, te, adv[j]);
+  const int64_t wid = static_cast<int64_t>(blockIdx.x) * (kThreads / 32) + (threadIdx.x >> 5);
+  if constexpr (!kFlat) {
+    for (int64_t j = wid; j < n_traj; j += nw) {
+      int64_t ts = traj_offsets[j], te = traj_offsets[j + 1];
+      ts = ts < 0 ? 0 : ts;
+      te = te > n_tokens ? n_tokens : te;
+      if (te > ts) stream_trajectory(ts, te, adv[j]);
+    }
+  } else {
+    const int64_t lo_c = lo < 0 ? 0 : lo, hi_c = hi > n_tokens ? n_tokens : hi;
+    const int64_t per = hi_c > lo_c ? ((hi_c - lo_c + nw - 1) / nw + 3) & ~int64_t{3} : 0;
+    const int64_t a = lo_c + per * wid;
+    const int64_t b = a + per < hi_c ? a + per : hi_c;
+    if (a < b) {
+      int64_t j = find_traj(traj_offsets, n_traj, a, lane);
+      int64_t j0 = j;
+      int64_t wo = traj_offsets[j0 + lane < n_traj ? j0 + lane : n_traj];
+      float wa = adv[j0 + lane < n_traj ? j0 + lane : n_traj - 1];
+      while (j < n_traj) {
+        if (j - j0 == 31) {   // lane 31 holds only the end of the window's last trajectory
+          j0 = j;
+          wo = traj_offsets[j0 + lane < n_traj ? j0 + lane : n_traj];
+          wa = adv[j0 + lane < n_traj ? j0 + lane : n_traj - 1];
+        }
+        const int i = static_cast<int>(j - j0);
+        const int64_t ts = __shfl_sync(0xffffffffu, wo, i);
+        const int64_t te = __shfl_sync(0xffffffffu, wo, i + 1);
+        if (ts >= b) break;
+        const float A = __shfl_sync(0xffffffffu, wa, i);
+        const int64_t ps = ts > a ? ts : a, pe = te < b ? te : b;
+        if (ps < pe) stream_trajectory(ps, pe, A);
+        ++j;
+      }
+    }
   }
-  const float s0 = block_sum_f(acc.obj, red);
-  const float s1 = block_sum_f(static_cast<float>(ntok), red);
-  const float s2 = block_sum_f(acc.clipped, red);
-  const float s3 = block_sum_f(acc.ratio, red);
+  float sf[4] = {acc.obj, static_cast<float>(ntok), acc.clipped, acc.ratio};
+  block_sum4(sf, red);
   // The last block to finish folds every block's partial sums in double, in
   // a fixed order (thread i takes blocks i, i + 256, ...; then a fixed
   // tree), so the result does not depend on which block that is.
   if (threadIdx.x == 0) {
-    partial[blockIdx.x] = Sums{s0, s1, s2, s3};
+    partial[blockIdx.x] = Sums{sf[0], sf[1], sf[2], sf[3]};
     __threadfence();
     s_last = atomicAdd(done, 1u) == gridDim.x - 1;
   }
   __syncthreads();
   if (!s_last) return;
   __threadfence();
-  double o = 0.0, t = 0.0, c = 0.0, r = 0.0;
+  double sd[4] = {0.0, 0.0, 0.0, 0.0};
   for (int b = threadIdx.x; b < static_cast<int>(gridDim.x); b += kThreads) {
-    o += __ldcg(&partial[b].obj);
-    t += __ldcg(&partial[b].tokens);
-    c += __ldcg(&partial[b].clipped);
-    r += __ldcg(&partial[b].ratio);
+    sd[0] += __ldcg(&partial[b].obj);
+    sd[1] += __ldcg(&partial[b].tokens);
+    sd[2] += __ldcg(&partial[b].clipped);
+    sd[3] += __ldcg(&partial[b].ratio);
   }
-  o = block_sum(o, red_d);
-  t = block_sum(t, red_d);
-  c = block_sum(c, red_d);
-  r = block_sum(r, red_d);
+  block_sum4(sd, red_d);
+  const double o = sd[0], t = sd[1], c = sd[2], r = sd[3];
   if (threadIdx.x == 0) {
     const bool any = t > 0.0;
     stats[0] = any ? static_cast<float>(-o / t) : 0.f;
@@ -328,19 +369,25 @@ extern "C" hdl_status hdl_grpo_loss(const float* logp_new, const float* logp_old
       reinterpret_cast<uint8_t*>(counts) + align_up(kMaxBlocks * sizeof(unsigned long long), 256));
   const bool vec = n_tokens > 0 && aligned_to(logp_new, 16) && aligned_to(logp_old, 16) &&
                    aligned_to(mask, 4) && (grad == nullptr || aligned_to(grad, 16));
-  auto tok = vec ? grpo_token_kernel<true> : grpo_token_kernel<false>;
   // persistent grids: as many blocks as are resident at once (<= kMaxBlocks)
   int per_sm = 0;
-  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, tok, kThreads, 0) != cudaSuccess ||
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, grpo_token_kernel<true, false>,
+                                                    kThreads, 0) != cudaSuccess ||
       per_sm <= 0)
     per_sm = 4;
   const int64_t cap = static_cast<int64_t>(per_sm) * sms;
-  int64_t want = ceil_div(n_traj, kThreads / 32);          // one warp per trajectory
+  // fewer trajectories than about two rounds of the resident warps: equal
+  // token ranges per warp instead of one warp per trajectory
+  const bool flat = n_tokens > 0 && int64_t{n_traj} < 2 * cap * (kThreads / 32);
+  auto tok = vec ? (flat ? grpo_token_kernel<true, true> : grpo_token_kernel<true, false>)
+                 : (flat ? grpo_token_kernel<false, true> : grpo_token_kernel<false, false>);
+  // flat: at least 2048 tokens per block, up to every resident warp
+  int64_t want = flat ? ceil_div(n_tokens, int64_t{2048}) : ceil_div(n_traj, kThreads / 32);
   int blocks = static_cast<int>(want < cap ? want : cap);
   if (blocks > kMaxBlocks) blocks = kMaxBlocks;
   if (blocks < 1) blocks = 1;
-  // pass 0 sized by its own work: 64 KiB of mask or 8 groups per block
-  want = ceil_div(n_tokens, int64_t{65536});
+  // pass 0 sized by its own work: 16 KiB of mask or 8 groups per block
+  want = ceil_div(n_tokens, int64_t{16384});
   const int64_t gwant = ceil_div(n_groups, kThreads / 32);
   if (gwant > want) want = gwant;
   int prep = static_cast<int>(want < 4 * sms ? want : 4 * sms);
