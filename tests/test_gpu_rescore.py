@@ -46,6 +46,7 @@ SHAPES = [
     (1000, 1024, 8192, "bf16"),
     (200, 256, 5000, "f32"),   # tf32 path
     (513, 64, 4096, "f32"),
+    (3, 256, 152064, "bf16"),  # decode-like: a few tokens, a full vocabulary (one tile per unit)
 ]
 
 
