@@ -1,6 +1,7 @@
-"""The HDL step (re-scoring, selection, allocation, masks) captured in one
-CUDA graph and replayed gives bit for bit what the eager calls give: every
-call is capture-safe (kernel launches and one memset, no host sync)."""
+"""The HDL step (re-scoring, selection, allocation, masks) and the GRPO update
+captured in CUDA graphs and replayed give bit for bit what the eager calls
+give: every call is capture-safe (kernel launches and one memset, no host
+sync)."""
 import pytest
 import torch
 
@@ -60,3 +61,44 @@ def test_step_in_cuda_graph(hdl):
     assert hdl.hdl_device_status(ws)[0] == hdl.HDL_OK
     for a, b in zip(eager, (lp0, lp1, de, bp, ns, bd, cb, mask)):
         assert torch.equal(a, b) or torch.equal(torch.nan_to_num(a, nan=-7), torch.nan_to_num(b, nan=-7))
+
+
+@pytest.mark.parametrize("J,L", [(16, 3000), (12000, 40)])   # the flat and the per-trajectory pass
+def test_grpo_in_cuda_graph(hdl, J, L):
+    """The GRPO update captured in a CUDA graph and replayed several times
+    gives the eager call's advantages, gradient and statistics bit for bit
+    (its completion counter is re-armed by the first kernel of every replay)."""
+    g = torch.Generator(device="cuda").manual_seed(J)
+    T = J * L
+    lpo = -torch.rand(T, generator=g, device="cuda") * 3
+    lpn = lpo + torch.randn(T, generator=g, device="cuda") * 0.3
+    m = (torch.rand(T, generator=g, device="cuda") < 0.7).to(torch.uint8)
+    toffs = torch.arange(0, T + 1, L, dtype=torch.int64, device="cuda")
+    R = torch.rand(J, generator=g, device="cuda")
+    goffs = torch.arange(0, J + 1, 16, dtype=torch.int32, device="cuda")
+    adv = torch.empty(J, device="cuda")
+    grad = torch.empty(T, device="cuda")
+    st = torch.empty(4, device="cuda")
+    ws = torch.empty(hdl.hdl_grpo_loss_workspace_bytes(), dtype=torch.uint8, device="cuda")
+
+    def call(stream):
+        hdl.hdl_grpo_loss(lpn, lpo, m, toffs, R, goffs, advantages=adv, grad=grad, stats=st,
+                          workspace=ws, stream=stream)
+
+    call(torch.cuda.current_stream())
+    torch.cuda.synchronize()
+    eager = [t.clone() for t in (adv, grad, st)]
+    for t in (adv, grad, st):
+        t.fill_(float("nan"))
+    side = torch.cuda.Stream()
+    side.wait_stream(torch.cuda.current_stream())
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.stream(side):
+        with torch.cuda.graph(graph, stream=side):
+            call(side)
+    torch.cuda.current_stream().wait_stream(side)
+    for _ in range(4):
+        graph.replay()
+    torch.cuda.synchronize()
+    for a, b in zip(eager, (adv, grad, st)):
+        assert torch.equal(a, b)
