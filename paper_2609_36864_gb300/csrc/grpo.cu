@@ -345,6 +345,7 @@ extern "C" hdl_status hdl_grpo_loss(const float* logp_new, const float* logp_old
                                     float* advantages, float* grad, float* stats,
                                     void* workspace, size_t workspace_bytes,
                                     void* cuda_stream) {
+  HostRange range_("hdl_grpo_loss");
   if (n_tokens < 0 || n_traj < 0 || n_groups < 0) return HDL_ERR_INVALID_ARG;
   if (!(eps_low >= 0.f && eps_low < 1.f && eps_high >= 0.f)) return HDL_ERR_INVALID_ARG;
   if (!stats || (n_traj > 0 && !advantages) || (n_groups > 0 && (!rewards || !group_offsets)))

@@ -167,6 +167,7 @@ extern "C" hdl_status hdl_assign_continuations(const int32_t* n_selected,
                                                int32_t k, const int32_t* conts_per_root,
                                                int32_t extra_to_higher, int32_t* cont_branch,
                                                int64_t n_cont_capacity, void* cuda_stream) {
+  HostRange range_("hdl_assign_continuations");
   if (n_roots < 0 || k < 0 || n_cont_capacity < 0) return HDL_ERR_INVALID_ARG;
   if (k > 16) return HDL_ERR_UNSUPPORTED;
   if (n_roots == 0 || n_cont_capacity == 0) return HDL_OK;
@@ -184,6 +185,7 @@ extern "C" hdl_status hdl_assign_continuations(const int32_t* n_selected,
 extern "C" hdl_status hdl_suffix_mask(const int32_t* cont_branch, const int64_t* cont_offsets,
                                       int32_t n_cont, const uint8_t* cont_valid, uint8_t* mask,
                                       int64_t mask_len, void* cuda_stream) {
+  HostRange range_("hdl_suffix_mask");
   if (n_cont < 0 || mask_len < 0) return HDL_ERR_INVALID_ARG;
   if (n_cont == 0 || mask_len == 0) return HDL_OK;
   if (!cont_branch || !cont_offsets || !mask) return HDL_ERR_INVALID_ARG;

@@ -747,6 +747,7 @@ extern "C" hdl_status hdl_rescore_ex(const void* h_orig, const void* h_hind,
                                      float* delta, const hdl_rescore_opts* opts,
                                      void* workspace, size_t workspace_bytes,
                                      void* cuda_stream) {
+  HostRange range_("hdl_rescore_ex");
   const hdl_status sh = check_shape(n_tokens, d, vocab, dt);
   if (sh != HDL_OK) return sh;
   if (n_tokens == 0) return HDL_OK;
@@ -836,6 +837,7 @@ extern "C" hdl_status hdl_rescore(const void* h_orig, const void* h_hind, const 
 
 extern "C" hdl_status hdl_device_status(const void* workspace, size_t workspace_bytes,
                                         void* cuda_stream, uint32_t* raw_word) {
+  HostRange range_("hdl_device_status");
   if (!workspace || workspace_bytes < sizeof(uint32_t)) return HDL_ERR_INVALID_ARG;
   if (cudaStreamSynchronize(as_stream(cuda_stream)) != cudaSuccess) return HDL_ERR_CUDA;
   uint32_t word = 0;
@@ -880,6 +882,7 @@ extern "C" hdl_status hdl_rescore_noalloc(const void* h_orig, const void* h_hind
                                           int32_t vocab, float* logp_orig, float* logp_hind,
                                           float* delta, const void** scratch_out,
                                           void* cuda_stream) {
+  HostRange range_("hdl_rescore_noalloc");
   const hdl_status sh = check_shape(n_tokens, d, vocab, dt);
   if (sh != HDL_OK) return sh;
   if (n_tokens == 0) return HDL_OK;
@@ -907,6 +910,7 @@ extern "C" hdl_status hdl_rescore_shard(const void* h_orig, const void* h_hind,
                                         int32_t vocab_shard, int32_t vocab_offset, float* stats,
                                         void* workspace, size_t workspace_bytes,
                                         void* cuda_stream) {
+  HostRange range_("hdl_rescore_shard");
   const hdl_status sh = check_shape(n_tokens, d, vocab_shard, dt);
   if (sh != HDL_OK) return sh;
   if (vocab_offset < 0) return HDL_ERR_INVALID_ARG;
@@ -968,6 +972,7 @@ extern "C" hdl_status hdl_merge_vocab_shards(const float* stats, int32_t n_shard
                                              float* logp_hind, float* delta,
                                              float* entropy_orig, float* entropy_hind,
                                              void* cuda_stream) {
+  HostRange range_("hdl_merge_vocab_shards");
   if (n_shards <= 0 || n_tokens < 0) return HDL_ERR_INVALID_ARG;
   if (n_tokens == 0) return HDL_OK;
   if (!stats || !logp_orig || !logp_hind) return HDL_ERR_INVALID_ARG;

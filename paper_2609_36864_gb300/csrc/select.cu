@@ -588,6 +588,7 @@ extern "C" hdl_status hdl_select_branches(const float* delta, const uint8_t* val
                                           const hdl_select_opts* opts, int32_t* branch_pos,
                                           int32_t* n_selected, float* branch_delta,
                                           void* cuda_stream) {
+  HostRange range_("hdl_select_branches");
   if (n_roots < 0 || n_tokens < 0 || k < 0) return HDL_ERR_INVALID_ARG;
   if (k > kMaxK) return HDL_ERR_UNSUPPORTED;
   hdl_select_opts o{0, 0, 0, 0};
