@@ -223,7 +223,7 @@ HDL_API hdl_status hdl_grpo_loss(const float* logp_new, const float* logp_old,
  * memory is owned by a pooling allocator, where a cudaMalloc can fail or
  * fragment the pool; and latency-critical loops, where cudaMalloc/cudaFree
  * can synchronise the device.  Instead of a caller-provided workspace it uses
- * one file-scope device array of HDL_STATIC_SCRATCH_BYTES (16 MiB) that every
+ * one file-scope device array of HDL_STATIC_SCRATCH_BYTES (64 MiB) that every
  * GPU which loads the library holds until the process exits.  It calls no
  * cudaMalloc, cudaFree or allocating library routine.
  *
@@ -231,8 +231,8 @@ HDL_API hdl_status hdl_grpo_loss(const float* logp_new, const float* logp_old,
  *   - Returns HDL_ERR_UNSUPPORTED, before launching anything, when the
  *     problem needs more than HDL_STATIC_SCRATCH_BYTES of scratch, i.e. when
  *     hdl_rescore_workspace_bytes(n_tokens, d, vocab, dt) exceeds it
- *     (e.g. at vocab = 152064 about 27,000 tokens fit; at vocab = 32000
- *     about 123,000).
+ *     (e.g. at d = 3584, vocab = 152064 about 28,000 tokens fit; at d = 2048,
+ *     vocab = 32000 about 250,000).
  *   - The first call on a device looks up the array's device address (with
  *     that device current) and caches it; make that first call before any
  *     stream capture.
@@ -243,7 +243,7 @@ HDL_API hdl_status hdl_grpo_loss(const float* logp_new, const float* logp_old,
  *   - scratch_out (host pointer, may be NULL) receives the array's device
  *     address, which hdl_device_status() accepts (with
  *     HDL_STATIC_SCRATCH_BYTES) to read the device status of the last call. */
-#define HDL_STATIC_SCRATCH_BYTES ((size_t)16 << 20)
+#define HDL_STATIC_SCRATCH_BYTES ((size_t)64 << 20)
 
 HDL_API hdl_status hdl_rescore_noalloc(const void* h_orig, const void* h_hind,
                                const void* w_lmhead, hdl_dtype dt,

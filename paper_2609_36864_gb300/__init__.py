@@ -29,7 +29,7 @@ __all__ = [
 HDL_OK, HDL_ERR_INVALID_ARG, HDL_ERR_UNSUPPORTED, HDL_ERR_WORKSPACE = 0, 1, 2, 3
 HDL_ERR_CUDA, HDL_ERR_TIMEOUT, HDL_ERR_BAD_TARGET = 4, 5, 6
 HDL_BF16, HDL_F32 = 0, 1
-HDL_STATIC_SCRATCH_BYTES = 16 << 20
+HDL_STATIC_SCRATCH_BYTES = 64 << 20
 
 _PKG = os.path.dirname(os.path.abspath(__file__))
 _lib = None
@@ -345,7 +345,7 @@ def hdl_rescore_noalloc(h_orig, h_hind, w_lmhead, targets, logp_orig, logp_hind,
                         stream=None):
     """hdl_rescore without a workspace, for callers that must not allocate
     device memory while they run (inference-runtime plugins, pool-owned
-    device memory, latency-critical loops).  Scratch is one static 16 MiB
+    device memory, latency-critical loops).  Scratch is one static 64 MiB
     device array shared by all calls: calls that overlap on the GPU race, and
     problems needing more scratch are rejected (HDL_ERR_UNSUPPORTED).  Every
     output tensor must be given; nothing is allocated here either.  Returns

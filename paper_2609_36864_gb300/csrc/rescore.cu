@@ -50,6 +50,8 @@ constexpr int kBN = 256;             // vocabulary columns per tile
 constexpr int kRowBytes = 128;       // K bytes per stage (one 128-byte swizzle row)
 constexpr int kMaxTilesPerChunk = 16;  // up to 4096 vocabulary entries per unit
 constexpr int64_t kMinUnits = 1216;     // 8 x 152: chunks shrink until this many units
+constexpr double kL2Budget = 80e6;      // bytes of L2 the running units' tiles may use
+constexpr int kPairsInFlight = 76;      // CTA pairs resident on 152 SMs
 #ifndef HDL_GROUP_M
 #define HDL_GROUP_M 32
 #endif
@@ -565,6 +567,30 @@ struct Geometry {
   size_t zt_off, part_off, part_t_off, total, total_ent;
 };
 
+// M-tiles per rasterisation group: HDL_GROUP_M (an even number in [2, 512])
+// overrides kGroupM for tuning; it also sets the vocabulary chunk (see
+// geometry), so results agree to rounding.
+int rescore_group_m() {
+  static const int g = [] {
+    const char* e = std::getenv("HDL_GROUP_M");
+    const int v = e ? std::atoi(e) : 0;
+    return (v >= 2 && v <= 512 && v % 2 == 0) ? v : kGroupM;
+  }();
+  return g;
+}
+
+// HDL_CHUNK_TILES (1 ... 16) caps the vocabulary tiles per chunk, for tuning;
+// results agree to rounding (the chunks' partial sums are merged in another
+// grouping).
+int chunk_tiles_override() {
+  static const int v = [] {
+    const char* e = std::getenv("HDL_CHUNK_TILES");
+    const int t = e ? std::atoi(e) : 0;
+    return (t >= 1 && t <= kMaxTilesPerChunk) ? t : 0;
+  }();
+  return v;
+}
+
 Geometry geometry(int64_t n, int32_t d, int32_t vocab, hdl_dtype dt) {
   Geometry g{};
   g.n = n;
@@ -573,11 +599,28 @@ Geometry geometry(int64_t n, int32_t d, int32_t vocab, hdl_dtype dt) {
   g.num_m_ctx = static_cast<int>(ceil_div(n, kBM));
   g.num_m = 2 * g.num_m_ctx;
   g.num_vt = static_cast<int>(ceil_div(vocab, kBN));
-  // Small problems split the vocabulary finer so that every SM gets work.
+  // The chunk: the largest power of two (<= 16 tiles) for which the tiles the
+  // concurrently running units touch stay within kL2Budget of the 126 MB L2
+  // -- the H tiles of one rasterisation group (group_m x 128 rows) plus the W
+  // tiles of the chunks in flight (one chunk per group_m / 2 running pairs,
+  // 76 pairs on 152 SMs).  Past that, W tiles are evicted before the group's
+  // last pairs use them: on the code-shaped workload 4-tile chunks read 90 GB
+  // from DRAM per launch instead of 156 GB and run 2.5 % faster, agent-shaped
+  // (d = 5120) 2-tile chunks 9 % faster, and working sets just above the
+  // budget (92-120 MB) were the slowest of all.
+  const double row = static_cast<double>(d) * g.esize;
+  const int gm = rescore_group_m();
+  const double h_bytes = gm * static_cast<double>(kBM) * row;
+  const double chunks_in_flight = 2.0 * kPairsInFlight / gm;
   g.tiles_per_chunk = kMaxTilesPerChunk;
+  while (g.tiles_per_chunk > 1 &&
+         h_bytes + chunks_in_flight * g.tiles_per_chunk * kBN * row > kL2Budget)
+    g.tiles_per_chunk /= 2;
+  // Small problems split the vocabulary finer so that every SM gets work.
   while (g.tiles_per_chunk > 1 &&
          static_cast<int64_t>(g.num_m) * ceil_div(g.num_vt, g.tiles_per_chunk) < kMinUnits)
     g.tiles_per_chunk /= 2;
+  if (const int t = chunk_tiles_override(); t > 0 && t < g.tiles_per_chunk) g.tiles_per_chunk = t;
   g.num_chunks = static_cast<int>(ceil_div(g.num_vt, g.tiles_per_chunk));
   g.num_units = static_cast<int64_t>(g.num_m) * g.num_chunks;
   g.zt_off = 256;
@@ -700,16 +743,6 @@ int rescore_mode() {
   return mode;
 }
 
-// M-tiles per rasterisation group: HDL_GROUP_M (an even number in [2, 512])
-// overrides kGroupM for tuning; results do not depend on it.
-int rescore_group_m() {
-  static const int g = [] {
-    const char* e = std::getenv("HDL_GROUP_M");
-    const int v = e ? std::atoi(e) : 0;
-    return (v >= 2 && v <= 512 && v % 2 == 0) ? v : kGroupM;
-  }();
-  return g;
-}
 
 hdl_status check_shape(int64_t n_tokens, int32_t d, int32_t vocab, hdl_dtype dt) {
   if (n_tokens < 0 || d <= 0 || vocab <= 0) return HDL_ERR_INVALID_ARG;

@@ -53,14 +53,24 @@ def test_abi_version_and_names(L):
     assert hdl.hdl_status_string(99) == "HDL_ERR_UNKNOWN"
 
 
-def _ws_formula(n, d, V):
-    """status (256 B) + target logits + per-(chunk, row) partials; the chunk
-    shrinks from 16 vocabulary tiles until there are >= 1216 work units."""
+def _chunk_tiles(n, d, V, esize):
+    """Vocabulary tiles per chunk: from 16, halved while the H tiles of a group
+    of 32 M-tiles plus the W tiles of the 76 / 16 chunks in flight exceed
+    80 MB, then while there are fewer than 1216 work units."""
     cdiv = lambda a, b: -(-a // b)
     num_m, nvt, tpc = 2 * cdiv(n, 128), cdiv(V, 256), 16
+    row = d * esize
+    while tpc > 1 and 32 * 128 * row + (2 * 76 / 32) * tpc * 256 * row > 80e6:
+        tpc //= 2
     while tpc > 1 and num_m * cdiv(nvt, tpc) < 1216:
         tpc //= 2
-    chunks = cdiv(nvt, tpc)
+    return tpc
+
+
+def _ws_formula(n, d, V, esize=2):
+    """status (256 B) + target logits + per-(chunk, row) partials."""
+    cdiv = lambda a, b: -(-a // b)
+    chunks = cdiv(cdiv(V, 256), _chunk_tiles(n, d, V, esize))
     zt = cdiv(2 * n * 4, 256) * 256
     return 256 + zt + chunks * 2 * n * 8
 
@@ -70,8 +80,8 @@ def _ws_formula(n, d, V):
                                    (5, 128, 4097), (8192, 4096, 32000), (1000, 64, 152064)])
 def test_workspace_bytes(L, n, d, V):
     import paper_2609_36864_gb300 as hdl
-    assert hdl.hdl_rescore_workspace_bytes(n, d, V, hdl.HDL_BF16) == _ws_formula(n, d, V)
-    assert hdl.hdl_rescore_workspace_bytes(n, d, V, hdl.HDL_F32) == _ws_formula(n, d, V)
+    assert hdl.hdl_rescore_workspace_bytes(n, d, V, hdl.HDL_BF16) == _ws_formula(n, d, V, 2)
+    assert hdl.hdl_rescore_workspace_bytes(n, d, V, hdl.HDL_F32) == _ws_formula(n, d, V, 4)
 
 
 def test_workspace_bytes_rejects_bad_shapes(L):
@@ -162,10 +172,7 @@ def test_rescore_ex_options_and_workspace(L):
     assert hdl.hdl_rescore_ex_workspace_bytes(n, d, V) == base
     ent = hdl.hdl_rescore_ex_workspace_bytes(n, d, V, entropy=True)
     cdiv = lambda a, b: -(-a // b)
-    num_m, nvt, tpc = 2 * cdiv(n, 128), cdiv(V, 256), 16
-    while tpc > 1 and num_m * cdiv(nvt, tpc) < 1216:
-        tpc //= 2
-    assert ent == cdiv(base, 256) * 256 + cdiv(nvt, tpc) * 2 * n * 4
+    assert ent == cdiv(base, 256) * 256 + cdiv(cdiv(V, 256), _chunk_tiles(n, d, V, 2)) * 2 * n * 4
     o = hdl._RescoreOpts(None, None, 0, 2, 0)          # unknown fault bit
     assert L.hdl_rescore_ex(P, P, P, 0, P, 16, 64, 100, P, P, None, ctypes.byref(o), P,
                             1 << 40, None) == 1

@@ -5,7 +5,7 @@ callbacks of inference runtimes forbid it, processes whose device memory is
 owned by a pooling allocator risk failure or fragmentation, and
 latency-critical loops cannot afford the device synchronisation that
 cudaMalloc/cudaFree may cause.  hdl_rescore_noalloc serves them from one
-static 16 MiB device array.  These tests check that two calls in a row, on
+static 64 MiB device array.  These tests check that two calls in a row, on
 different inputs, give what hdl_rescore gives on the same inputs (within the
 log-probability tolerance of the parity tests), and that problems needing
 more scratch than the array holds are refused before anything runs.
@@ -81,7 +81,7 @@ def test_noalloc_refuses_oversized_problems(hdl):
     """Refused on the host, before any CUDA call (runs without a GPU)."""
     L = hdl.lib()
     P = ctypes.c_void_p(0x10000)
-    n = 100_000   # at V = 152064 this needs ~62 MB of scratch
+    n = 100_000   # at d = 4096, V = 152064 this needs ~228 MiB of scratch
     assert hdl.hdl_rescore_workspace_bytes(n, 4096, 152064) > hdl.HDL_STATIC_SCRATCH_BYTES
     code = L.hdl_rescore_noalloc(P, P, P, 0, P, n, 4096, 152064, P, P, None, None, None)
     assert code == hdl.HDL_ERR_UNSUPPORTED
