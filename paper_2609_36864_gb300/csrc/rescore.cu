@@ -50,7 +50,7 @@ constexpr int kBN = 256;             // vocabulary columns per tile
 constexpr int kRowBytes = 128;       // K bytes per stage (one 128-byte swizzle row)
 constexpr int kMaxTilesPerChunk = 16;  // up to 4096 vocabulary entries per unit
 constexpr int64_t kMinUnits = 1216;     // 8 x 152: chunks shrink until this many units
-constexpr double kL2Budget = 80e6;      // bytes of L2 the running units' tiles may use
+constexpr double kL2Budget = 75e6;      // bytes of L2 the running units' tiles may use
 constexpr int kPairsInFlight = 76;      // CTA pairs resident on 152 SMs
 #ifndef HDL_GROUP_M
 #define HDL_GROUP_M 32
@@ -607,7 +607,7 @@ Geometry geometry(int64_t n, int32_t d, int32_t vocab, hdl_dtype dt) {
   // last pairs use them: on the code-shaped workload 4-tile chunks read 90 GB
   // from DRAM per launch instead of 156 GB and run 2.5 % faster, agent-shaped
   // (d = 5120) 2-tile chunks 9 % faster, and working sets just above the
-  // budget (92-120 MB) were the slowest of all.
+  // budget (76-120 MB) were the slowest of all.
   const double row = static_cast<double>(d) * g.esize;
   const int gm = rescore_group_m();
   const double h_bytes = gm * static_cast<double>(kBM) * row;
