@@ -8,13 +8,13 @@
 // running (max, sum of exponentials) per row, picking the target logit out of
 // the tile that holds it.
 //
-// Work unit = (M-tile of 128 rows of one context, vocabulary chunk of
-// up to 16 256-wide tiles).  Each unit writes one partial (max, sum)
-// per row; a second, tiny kernel merges the chunks, forms both log-probs,
-// |Delta| and, when asked, the entropies.  Splitting the vocabulary keeps the set of tiles that the ~150
-// concurrently running units touch small enough to stay in L2 (grouped
-// rasterisation: 32 M-tiles x a few chunks at a time), instead of every
-// CTA streaming its own 128 x d slice of H for the whole vocabulary.
+// Work unit = (M-tile of 128 rows of one context, vocabulary chunk of up to
+// 16 256-wide tiles).  Each unit writes one partial (max, sum) per row; a
+// second, small kernel merges the chunks, forms both log-probs, |Delta| and,
+// when asked, the entropies.  Units are rasterised in groups of 32 M-tiles x
+// the chunks, and the chunk is sized (see geometry) so that the H and W tiles
+// the ~150 concurrently running units touch stay in L2 -- W is then streamed
+// from DRAM once per group instead of once per M-tile.
 //
 // Roles inside a CTA of 192 threads (shown for the single-CTA organisation;
 // Cfg below describes the CTA-pair ones, the default):
