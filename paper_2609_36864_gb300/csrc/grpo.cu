@@ -5,13 +5,14 @@
 //
 // Two HBM-bound launches over the packed tokens: (0) the group advantages
 // and an exact integer count of the masked tokens per block (1 byte per
-// token, 16-byte loads); (1) one warp per trajectory -- its advantage a
-// warp-uniform scalar, its tokens streamed with 16-byte loads -- writes the
-// final gradient (the denominator, folded from the counts, is known up
-// front) and per-block fp32 sums; the last block to finish folds the block
-// sums in double precision in a fixed order, so the loss does not depend on
-// the timing of atomics.  The GPU's fp64 rate is low, so nothing per token
-// runs in double.
+// token, 16-byte loads); (1) the token pass -- one warp per trajectory when
+// there are many, equal token ranges per warp when there are few; either way
+// the advantage is a warp-uniform scalar per trajectory and the tokens are
+// streamed with 16-byte loads -- writes the final gradient (the denominator,
+// folded from the counts, is known up front) and per-block fp32 sums; the
+// last block to finish folds the block sums in double precision in a fixed
+// order, so the loss does not depend on the timing of atomics.  The GPU's
+// fp64 rate is low, so nothing per token runs in double.
 #include <cuda_runtime.h>
 
 #include <cstdint>
