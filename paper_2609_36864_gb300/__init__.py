@@ -132,23 +132,50 @@ def _ptr(t: Optional[torch.Tensor]):
     return None if t is None else ctypes.c_void_p(t.data_ptr())
 
 
-def _stream(stream) -> ctypes.c_void_p:
+def _stream(stream, device=None) -> ctypes.c_void_p:
     if stream is None:
-        stream = torch.cuda.current_stream()
+        stream = torch.cuda.current_stream(device)
     if isinstance(stream, torch.cuda.Stream):
         return ctypes.c_void_p(stream.cuda_stream)
     return ctypes.c_void_p(int(stream))
 
 
-def _dev(t: torch.Tensor, name: str, dtype=None):
+def _dev(t: torch.Tensor, name: str, dtype=None, numel: Optional[int] = None,
+         device: Optional[torch.device] = None):
+    """Check one tensor argument.  The C entry points receive raw pointers and
+    take every length from the scalar arguments, so a buffer shorter than
+    those lengths, or one on another device, must be caught here."""
     if not isinstance(t, torch.Tensor):
         raise TypeError(f"{name} must be a torch.Tensor")
     if t.device.type != "cuda":
         raise ValueError(f"{name} must be a CUDA tensor (got {t.device})")
+    if device is not None and t.device != device:
+        raise ValueError(f"{name} is on {t.device}, the other arguments on {device}")
     if not t.is_contiguous():
         raise ValueError(f"{name} must be contiguous")
     if dtype is not None and t.dtype != dtype:
         raise ValueError(f"{name} must be {dtype} (got {t.dtype})")
+    if numel is not None and t.numel() != numel:
+        raise ValueError(f"{name} must hold {numel} elements (got {t.numel()})")
+
+
+def _lm_inputs(h_orig, h_hind, w, targets, w_name="w_lmhead"):
+    """Validate the operands of a re-scoring call; returns (dtype code, N, d, V, device)."""
+    _dev(h_orig, "h_orig")
+    dev = h_orig.device
+    _dev(h_hind, "h_hind", device=dev)
+    _dev(w, w_name, device=dev)
+    _dev(targets, "targets", torch.int32, device=dev)
+    dt = _hdl_dtype(h_orig)
+    if h_hind.dtype != h_orig.dtype or w.dtype != h_orig.dtype:
+        raise ValueError(f"h_orig, h_hind and {w_name} must share one dtype")
+    if h_orig.dim() != 2 or w.dim() != 2:
+        raise ValueError(f"h_orig and {w_name} must be 2-D")
+    N, d = h_orig.shape
+    V = w.shape[0]
+    if h_hind.shape != (N, d) or w.shape != (V, d) or targets.shape != (N,):
+        raise ValueError(f"shape mismatch between h_orig, h_hind, {w_name}, targets")
+    return dt, N, d, V, dev
 
 
 def _hdl_dtype(t: torch.Tensor) -> int:
@@ -182,17 +209,7 @@ def hdl_rescore(h_orig, h_hind, w_lmhead, targets, logp_orig=None, logp_hind=Non
     allocated.  Asynchronous on ``stream``; device-side errors surface through
     :func:`hdl_device_status` on the returned workspace.
     """
-    for t, n in ((h_orig, "h_orig"), (h_hind, "h_hind"), (w_lmhead, "w_lmhead")):
-        _dev(t, n)
-    _dev(targets, "targets", torch.int32)
-    dt = _hdl_dtype(h_orig)
-    if h_hind.dtype != h_orig.dtype or w_lmhead.dtype != h_orig.dtype:
-        raise ValueError("h_orig, h_hind and w_lmhead must share one dtype")
-    N, d = h_orig.shape
-    V = w_lmhead.shape[0]
-    if h_hind.shape != (N, d) or w_lmhead.shape != (V, d) or targets.shape != (N,):
-        raise ValueError("shape mismatch between h_orig, h_hind, w_lmhead, targets")
-    dev = h_orig.device
+    dt, N, d, V, dev = _lm_inputs(h_orig, h_hind, w_lmhead, targets)
     if logp_orig is None:
         logp_orig = torch.empty(N, dtype=torch.float32, device=dev)
     if logp_hind is None:
@@ -200,16 +217,16 @@ def hdl_rescore(h_orig, h_hind, w_lmhead, targets, logp_orig=None, logp_hind=Non
     if delta is None and want_delta:
         delta = torch.empty(N, dtype=torch.float32, device=dev)
     for t, n in ((logp_orig, "logp_orig"), (logp_hind, "logp_hind")):
-        _dev(t, n, torch.float32)
+        _dev(t, n, torch.float32, N, dev)
     if delta is not None:
-        _dev(delta, "delta", torch.float32)
+        _dev(delta, "delta", torch.float32, N, dev)
     need = hdl_rescore_workspace_bytes(N, d, V, dt)
     if workspace is None:
         workspace = torch.empty(max(need, 256), dtype=torch.uint8, device=dev)
-    _dev(workspace, "workspace", torch.uint8)
+    _dev(workspace, "workspace", torch.uint8, device=dev)
     code = lib().hdl_rescore(_ptr(h_orig), _ptr(h_hind), _ptr(w_lmhead), dt, _ptr(targets),
                              N, d, V, _ptr(logp_orig), _ptr(logp_hind), _ptr(delta),
-                             _ptr(workspace), workspace.numel(), _stream(stream))
+                             _ptr(workspace), workspace.numel(), _stream(stream, dev))
     _check("hdl_rescore", code)
     return logp_orig, logp_hind, delta, workspace
 
@@ -236,19 +253,13 @@ def hdl_rescore_ex(h_orig, h_hind, w_lmhead, targets, logp_orig=None, logp_hind=
 
     Returns (logp_orig, logp_hind, delta, entropy_orig, entropy_hind, workspace).
     ``fault_inject`` is the library's test hook (see hdl_rescore_opts)."""
-    for t, n in ((h_orig, "h_orig"), (h_hind, "h_hind"), (w_lmhead, "w_lmhead")):
-        _dev(t, n)
-    _dev(targets, "targets", torch.int32)
-    dt = _hdl_dtype(h_orig)
-    N, d = h_orig.shape
-    V = w_lmhead.shape[0]
-    dev = h_orig.device
+    dt, N, d, V, dev = _lm_inputs(h_orig, h_hind, w_lmhead, targets)
 
     def out(t, want):
         if t is None and want:
             t = torch.empty(N, dtype=torch.float32, device=dev)
         if t is not None:
-            _dev(t, "output", torch.float32)
+            _dev(t, "output", torch.float32, N, dev)
         return t
     logp_orig, logp_hind = out(logp_orig, True), out(logp_hind, True)
     delta = out(delta, True)
@@ -258,20 +269,27 @@ def hdl_rescore_ex(h_orig, h_hind, w_lmhead, targets, logp_orig=None, logp_hind=
     need = int(lib().hdl_rescore_ex_workspace_bytes(N, d, V, dt, ctypes.byref(o)))
     if workspace is None:
         workspace = torch.empty(max(need, 256), dtype=torch.uint8, device=dev)
-    _dev(workspace, "workspace", torch.uint8)
+    _dev(workspace, "workspace", torch.uint8, device=dev)
     code = lib().hdl_rescore_ex(_ptr(h_orig), _ptr(h_hind), _ptr(w_lmhead), dt, _ptr(targets),
                                 N, d, V, _ptr(logp_orig), _ptr(logp_hind), _ptr(delta),
                                 ctypes.byref(o), _ptr(workspace), workspace.numel(),
-                                _stream(stream))
+                                _stream(stream, dev))
     _check("hdl_rescore_ex", code)
     return logp_orig, logp_hind, delta, entropy_orig, entropy_hind, workspace
 
 
-def hdl_device_status(workspace: torch.Tensor, stream=None):
-    """(status code, raw status word) of a re-scoring workspace; synchronises."""
+def hdl_device_status(workspace, stream=None):
+    """(status code, raw status word) of a re-scoring workspace; synchronises.
+
+    ``workspace`` is the workspace tensor of an earlier call, or the scratch
+    address that :func:`hdl_rescore_noalloc` returned."""
+    if isinstance(workspace, int):
+        ptr, size, dev = ctypes.c_void_p(workspace), HDL_STATIC_SCRATCH_BYTES, None
+    else:
+        _dev(workspace, "workspace", torch.uint8)
+        ptr, size, dev = _ptr(workspace), workspace.numel(), workspace.device
     raw = ctypes.c_uint32(0)
-    code = lib().hdl_device_status(_ptr(workspace), workspace.numel(), _stream(stream),
-                                   ctypes.byref(raw))
+    code = lib().hdl_device_status(ptr, size, _stream(stream, dev), ctypes.byref(raw))
     return int(code), int(raw.value)
 
 
@@ -280,22 +298,28 @@ def hdl_select_branches(delta, valid, root_offsets, k: int, min_gap: int = 0,
                         n_selected=None, branch_delta=None, want_delta=True, stream=None):
     """Top-k branch points per root; returns (branch_pos [R,k], n_selected [R], branch_delta)."""
     _dev(delta, "delta", torch.float32)
-    if valid is not None:
-        _dev(valid, "valid", torch.uint8)
-    _dev(root_offsets, "root_offsets", torch.int64)
-    R = root_offsets.numel() - 1
     dev = delta.device
+    if valid is not None:
+        _dev(valid, "valid", torch.uint8, delta.numel(), dev)
+    _dev(root_offsets, "root_offsets", torch.int64, device=dev)
+    R = root_offsets.numel() - 1
+    if R < 0:
+        raise ValueError("root_offsets needs n_roots + 1 entries")
     if branch_pos is None:
         branch_pos = torch.empty((R, k), dtype=torch.int32, device=dev)
     if n_selected is None:
         n_selected = torch.empty(R, dtype=torch.int32, device=dev)
     if branch_delta is None and want_delta:
         branch_delta = torch.empty((R, k), dtype=torch.float32, device=dev)
+    _dev(branch_pos, "branch_pos", torch.int32, R * k, dev)
+    _dev(n_selected, "n_selected", torch.int32, R, dev)
+    if branch_delta is not None:
+        _dev(branch_delta, "branch_delta", torch.float32, R * k, dev)
     opts = _SelectOpts(min_gap, gap_mode, lo, hi)
     code = lib().hdl_select_branches(_ptr(delta), _ptr(valid), delta.numel(),
                                      _ptr(root_offsets), R, k, ctypes.byref(opts),
                                      _ptr(branch_pos), _ptr(n_selected), _ptr(branch_delta),
-                                     _stream(stream))
+                                     _stream(stream, dev))
     _check("hdl_select_branches", code)
     return branch_pos, n_selected, branch_delta
 
@@ -303,19 +327,22 @@ def hdl_select_branches(delta, valid, root_offsets, k: int, min_gap: int = 0,
 def hdl_assign_continuations(n_selected, branch_pos, conts_per_root, extra_to_higher=True,
                              cont_branch=None, n_cont: Optional[int] = None, stream=None):
     """Root-relative branch position of every continuation (root-major)."""
-    _dev(n_selected, "n_selected", torch.int32)
     _dev(branch_pos, "branch_pos", torch.int32)
-    _dev(conts_per_root, "conts_per_root", torch.int32)
+    dev = branch_pos.device
+    if branch_pos.dim() != 2:
+        raise ValueError("branch_pos must be [n_roots, k]")
     R, k = branch_pos.shape
+    _dev(n_selected, "n_selected", torch.int32, R, dev)
+    _dev(conts_per_root, "conts_per_root", torch.int32, R, dev)
     if cont_branch is None:
         if n_cont is None:
             raise ValueError("give cont_branch or n_cont (the total continuation count)")
-        cont_branch = torch.empty(n_cont, dtype=torch.int32, device=branch_pos.device)
-    _dev(cont_branch, "cont_branch", torch.int32)
+        cont_branch = torch.empty(n_cont, dtype=torch.int32, device=dev)
+    _dev(cont_branch, "cont_branch", torch.int32, device=dev)
     code = lib().hdl_assign_continuations(_ptr(n_selected), _ptr(branch_pos), R, k,
                                           _ptr(conts_per_root), 1 if extra_to_higher else 0,
                                           _ptr(cont_branch), cont_branch.numel(),
-                                          _stream(stream))
+                                          _stream(stream, dev))
     _check("hdl_assign_continuations", code)
     return cont_branch
 
@@ -324,19 +351,22 @@ def hdl_suffix_mask(cont_branch, cont_offsets, cont_valid=None, mask=None,
                     mask_len: Optional[int] = None, stream=None):
     """Suffix-only loss mask of packed continuations (uint8)."""
     _dev(cont_branch, "cont_branch", torch.int32)
-    _dev(cont_offsets, "cont_offsets", torch.int64)
-    if cont_valid is not None:
-        _dev(cont_valid, "cont_valid", torch.uint8)
+    dev = cont_branch.device
     C = cont_branch.numel()
+    _dev(cont_offsets, "cont_offsets", torch.int64, C + 1, dev)
+    if cont_valid is not None:
+        _dev(cont_valid, "cont_valid", torch.uint8, device=dev)
     if mask is None:
         if mask_len is None:
             mask_len = cont_valid.numel() if cont_valid is not None else None
         if mask_len is None:
             raise ValueError("give mask, mask_len or cont_valid")
-        mask = torch.zeros(mask_len, dtype=torch.uint8, device=cont_branch.device)
-    _dev(mask, "mask", torch.uint8)
+        mask = torch.zeros(mask_len, dtype=torch.uint8, device=dev)
+    _dev(mask, "mask", torch.uint8, device=dev)
+    if cont_valid is not None and cont_valid.numel() != mask.numel():
+        raise ValueError("cont_valid and mask must have the same length")
     code = lib().hdl_suffix_mask(_ptr(cont_branch), _ptr(cont_offsets), C, _ptr(cont_valid),
-                                 _ptr(mask), mask.numel(), _stream(stream))
+                                 _ptr(mask), mask.numel(), _stream(stream, dev))
     _check("hdl_suffix_mask", code)
     return mask
 
@@ -351,19 +381,15 @@ def hdl_rescore_noalloc(h_orig, h_hind, w_lmhead, targets, logp_orig, logp_hind,
     output tensor must be given; nothing is allocated here either.  Returns
     the device address of the scratch array, which hdl_device_status()
     accepts."""
-    for t, n in ((h_orig, "h_orig"), (h_hind, "h_hind"), (w_lmhead, "w_lmhead")):
-        _dev(t, n)
-    _dev(targets, "targets", torch.int32)
+    dt, N, d, V, dev = _lm_inputs(h_orig, h_hind, w_lmhead, targets)
     for t, n in ((logp_orig, "logp_orig"), (logp_hind, "logp_hind")):
-        _dev(t, n, torch.float32)
+        _dev(t, n, torch.float32, N, dev)
     if delta is not None:
-        _dev(delta, "delta", torch.float32)
-    N, d = h_orig.shape
+        _dev(delta, "delta", torch.float32, N, dev)
     scratch = ctypes.c_void_p(0)
-    code = lib().hdl_rescore_noalloc(_ptr(h_orig), _ptr(h_hind), _ptr(w_lmhead),
-                                     _hdl_dtype(h_orig), _ptr(targets), N, d,
-                                     w_lmhead.shape[0], _ptr(logp_orig), _ptr(logp_hind),
-                                     _ptr(delta), ctypes.byref(scratch), _stream(stream))
+    code = lib().hdl_rescore_noalloc(_ptr(h_orig), _ptr(h_hind), _ptr(w_lmhead), dt,
+                                     _ptr(targets), N, d, V, _ptr(logp_orig), _ptr(logp_hind),
+                                     _ptr(delta), ctypes.byref(scratch), _stream(stream, dev))
     _check("hdl_rescore_noalloc", code)
     return scratch.value
 
@@ -380,21 +406,17 @@ def hdl_rescore_shard(h_orig, h_hind, w_shard, targets, vocab_offset: int, stats
     """Per-row statistics of one vocabulary shard of the LM head: a
     [2, n_tokens, 4] float tensor (max in log2 units, sum, target logit or NaN,
     entropy numerator), to be exchanged and merged by hdl_merge_vocab_shards."""
-    for t, n in ((h_orig, "h_orig"), (h_hind, "h_hind"), (w_shard, "w_shard")):
-        _dev(t, n)
-    _dev(targets, "targets", torch.int32)
-    dt = _hdl_dtype(h_orig)
-    N, d = h_orig.shape
-    Vs = w_shard.shape[0]
+    dt, N, d, Vs, dev = _lm_inputs(h_orig, h_hind, w_shard, targets, "w_shard")
     if stats is None:
-        stats = torch.empty((2, N, 4), dtype=torch.float32, device=h_orig.device)
-    _dev(stats, "stats", torch.float32)
+        stats = torch.empty((2, N, 4), dtype=torch.float32, device=dev)
+    _dev(stats, "stats", torch.float32, 2 * N * 4, dev)
     need = hdl_rescore_shard_workspace_bytes(N, d, Vs, dt)
     if workspace is None:
-        workspace = torch.empty(max(need, 256), dtype=torch.uint8, device=h_orig.device)
+        workspace = torch.empty(max(need, 256), dtype=torch.uint8, device=dev)
+    _dev(workspace, "workspace", torch.uint8, device=dev)
     code = lib().hdl_rescore_shard(_ptr(h_orig), _ptr(h_hind), _ptr(w_shard), dt, _ptr(targets),
                                    N, d, Vs, int(vocab_offset), _ptr(stats), _ptr(workspace),
-                                   workspace.numel(), _stream(stream))
+                                   workspace.numel(), _stream(stream, dev))
     _check("hdl_rescore_shard", code)
     return stats, workspace
 
@@ -413,12 +435,14 @@ def hdl_merge_vocab_shards(stats, logp_orig=None, logp_hind=None, delta=None,
     def out(t, want=True):
         if t is None and want:
             t = torch.empty(N, dtype=torch.float32, device=dev)
+        if t is not None:
+            _dev(t, "output", torch.float32, N, dev)
         return t
     logp_orig, logp_hind, delta = out(logp_orig), out(logp_hind), out(delta)
     entropy_orig, entropy_hind = out(entropy_orig, want_entropy), out(entropy_hind, want_entropy)
     code = lib().hdl_merge_vocab_shards(_ptr(stats), P, N, _ptr(logp_orig), _ptr(logp_hind),
                                         _ptr(delta), _ptr(entropy_orig), _ptr(entropy_hind),
-                                        _stream(stream))
+                                        _stream(stream, dev))
     _check("hdl_merge_vocab_shards", code)
     return logp_orig, logp_hind, delta, entropy_orig, entropy_hind
 
@@ -435,13 +459,15 @@ def hdl_grpo_loss(logp_new, logp_old, mask, traj_offsets, rewards, group_offsets
     Returns (advantages [J], grad [T] or None, stats [4] = loss, masked
     tokens, clipped fraction, mean ratio), all on the device."""
     _dev(logp_new, "logp_new", torch.float32)
-    _dev(logp_old, "logp_old", torch.float32)
-    _dev(mask, "mask", torch.uint8)
-    _dev(traj_offsets, "traj_offsets", torch.int64)
-    _dev(rewards, "rewards", torch.float32)
-    _dev(group_offsets, "group_offsets", torch.int32)
     dev = logp_new.device
     T, J, G = logp_new.numel(), traj_offsets.numel() - 1, group_offsets.numel() - 1
+    if J < 0 or G < 0:
+        raise ValueError("traj_offsets and group_offsets need count + 1 entries")
+    _dev(logp_old, "logp_old", torch.float32, T, dev)
+    _dev(mask, "mask", torch.uint8, T, dev)
+    _dev(traj_offsets, "traj_offsets", torch.int64, device=dev)
+    _dev(rewards, "rewards", torch.float32, J, dev)
+    _dev(group_offsets, "group_offsets", torch.int32, device=dev)
     if advantages is None:
         advantages = torch.zeros(J, dtype=torch.float32, device=dev)
     if grad is None and want_grad:
@@ -450,9 +476,14 @@ def hdl_grpo_loss(logp_new, logp_old, mask, traj_offsets, rewards, group_offsets
         stats = torch.empty(4, dtype=torch.float32, device=dev)
     if workspace is None:
         workspace = torch.empty(hdl_grpo_loss_workspace_bytes(), dtype=torch.uint8, device=dev)
+    _dev(advantages, "advantages", torch.float32, J, dev)
+    if grad is not None:
+        _dev(grad, "grad", torch.float32, T, dev)
+    _dev(stats, "stats", torch.float32, 4, dev)
+    _dev(workspace, "workspace", torch.uint8, device=dev)
     code = lib().hdl_grpo_loss(_ptr(logp_new), _ptr(logp_old), _ptr(mask), T, _ptr(traj_offsets),
                                J, _ptr(rewards), _ptr(group_offsets), G, float(eps_low),
                                float(eps_high), _ptr(advantages), _ptr(grad), _ptr(stats),
-                               _ptr(workspace), workspace.numel(), _stream(stream))
+                               _ptr(workspace), workspace.numel(), _stream(stream, dev))
     _check("hdl_grpo_loss", code)
     return advantages, grad, stats
