@@ -29,7 +29,11 @@ def _worker(rank, world, port, q):
     bench.barrier(w)
     t = bench.max_over_ranks(100.0 + 50.0 * rank, w)     # per-rank step times in ms
     spec = bench.spec_for("math", seed=r)
-    q.put((r, t, spec.seed, bench.aggregate_value(w, 1000, 10, t)))
+    # rank 1 alone saw a thermal slowdown: both ranks must take the timing again
+    clk = {"sm_mhz": 1900.0, "sm_max_mhz": 2070.0,
+           "reasons": ["sw_thermal_slowdown"] if r == 1 else []}
+    again = bench.max_over_ranks(float(bench.clock_suspect(clk)), w) > 0
+    q.put((r, t, spec.seed, bench.aggregate_value(w, 1000, 10, t), again))
     bench.barrier(w)
     dist.destroy_process_group()
 
@@ -50,8 +54,21 @@ def test_two_gloo_ranks():
     assert [x[1] for x in res] == [150.0, 150.0]          # slowest rank's time
     assert [x[2] for x in res] == [0, 1]                  # independent workloads
     assert res[0][3] == pytest.approx(2 * 1000 * 10 / 0.150)
+    assert [x[4] for x in res] == [True, True]            # re-measured on every rank
 
 
 def test_aggregate_value_single_rank():
     import bench
     assert bench.aggregate_value(1, 155979, 10, 2000.0) == pytest.approx(779895.0)
+
+
+def test_clock_suspect_rules():
+    import bench
+    ok = dict(sm_mhz=1580.0, sm_max_mhz=2070.0)
+    assert not bench.clock_suspect(dict(ok, reasons=["sw_power_cap"]))      # kept and noted
+    assert not bench.clock_suspect(dict(sm_mhz=2070.0, sm_max_mhz=2070.0, reasons=[]))
+    for r in bench.SLOWDOWNS:
+        assert bench.clock_suspect(dict(ok, reasons=[r, "sw_power_cap"]))
+    assert bench.clock_suspect(dict(ok, reasons=[]))      # low clock, no reason: a lock
+    assert not bench.clock_suspect({"sm_mhz": None, "sm_max_mhz": None,
+                                    "reasons": ["nvidia-smi unavailable"]})
