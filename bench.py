@@ -53,6 +53,12 @@ def parse():
                    help="print the comment-insensitive digest of csrc/FILE... and exit")
     p.add_argument("--micro", default=None, choices=["select", "mask", "grpo"],
                    help="bandwidth micro-benchmark of one HBM-bound kernel at a scaled size")
+    p.add_argument("--min-gap", type=int, default=0,
+                   help="--micro select: spacing rule distance (0 = plain top-k)")
+    p.add_argument("--gap-mode", type=int, default=0, choices=[0, 1],
+                   help="--micro select: 0 = greedy, 1 = drop-lower")
+    p.add_argument("--clustered", action="store_true",
+                   help="--micro select: lift 3 runs of 32 positions per root by 2.0")
     return p.parse_args()
 
 
@@ -526,13 +532,19 @@ def run_micro(args):
         delta = torch.rand(N, generator=g, device=dev)
         valid = (torch.rand(N, generator=g, device=dev) < 0.8).to(torch.uint8)
         offs = torch.arange(0, N + 1, T, dtype=torch.int64, device=dev)
+        if args.clustered:   # high scores in runs, where the spacing rule bites
+            first = torch.randint(0, T - 32, (R, 3), generator=g, device=dev) + offs[:-1, None]
+            run = (first[:, :, None] + torch.arange(32, device=dev)).reshape(-1)
+            delta[run] += 2.0
         bp = torch.empty((R, k), dtype=torch.int32, device=dev)
         ns = torch.empty(R, dtype=torch.int32, device=dev)
         bd = torch.empty((R, k), dtype=torch.float32, device=dev)
         fn = lambda: hdl.hdl_select_branches(delta, valid, offs, k, branch_pos=bp,
-                                             n_selected=ns, branch_delta=bd)
+                                             n_selected=ns, branch_delta=bd,
+                                             min_gap=args.min_gap, gap_mode=args.gap_mode)
         nbytes = N * 5 + 8 * (R + 1) + R * k * 8 + 4 * R
-        cfg = {"roots": R, "tokens_per_root": T, "k": k}
+        cfg = {"roots": R, "tokens_per_root": T, "k": k, "min_gap": args.min_gap,
+               "gap_mode": args.gap_mode, "clustered": args.clustered}
     elif args.micro == "mask":
         C, L = 32768, 4096
         offs = torch.arange(0, C * L + 1, L, dtype=torch.int64, device=dev)

@@ -20,12 +20,16 @@
 // and a bitonic merge with the list.  Many roots: S warps per root (usually
 // 1) in a persistent grid; few roots: 16 warps per root; the partial lists
 // of a root's warps are merged pairwise, a bitonic merge per level.
-// Spacing rule (min_gap > 0): select_spacing_kernel, one CTA per root --
-//   greedy (gap_mode 0): k rounds, each a full scan for the best key not
-//     within min_gap of an accepted point (the greedy walk of the ranked
-//     list accepts exactly these points in this order);
-//   drop-lower (gap_mode 1): plain top-k, then thread 0 walks the k points
-//     in rank order and keeps those not too close to a kept one.
+// Spacing rule (Section 4.4; min_gap > 0, |t - a| < min_gap counts as too
+// close):
+//   drop-lower (gap_mode 1): the plain top-k above, then the root's warp walks
+//     its k points in rank order and drops each one too close to a kept one;
+//   greedy (gap_mode 0): the greedy walk of the ranked list accepts, in
+//     rank order, each candidate not too close to an accepted one.  The same
+//     streaming kernel collects the 16 best candidates far enough from every
+//     point accepted so far, the root's warp walks them in rank order, and a
+//     new pass follows only while fewer than k are accepted and the pass came
+//     back full -- one to three passes on clustered scores, k at most.
 #include <cuda_runtime.h>
 
 #include <cstdint>
@@ -37,8 +41,6 @@
 namespace hdl {
 namespace {
 
-constexpr int kSelThreads = 512;
-constexpr int kSelWarps = kSelThreads / 32;
 constexpr int kMaxK = 16;
 
 __device__ __forceinline__ uint32_t score_order(float f) {
@@ -54,145 +56,6 @@ __device__ __forceinline__ uint64_t make_key(float score, int64_t t) {
 
 __device__ __forceinline__ int64_t key_pos(uint64_t key) {
   return static_cast<int64_t>(0xFFFFFFFFu - static_cast<uint32_t>(key & 0xFFFFFFFFu));
-}
-
-__device__ __forceinline__ uint64_t warp_max_u64(uint64_t v) {
-#pragma unroll
-  for (int o = 16; o >= 1; o >>= 1) {
-    const uint64_t w = __shfl_xor_sync(0xffffffffu, v, o);
-    v = w > v ? w : v;
-  }
-  return v;
-}
-
-// Block-wide max of one key per thread; every thread gets the result.
-__device__ __forceinline__ uint64_t block_max_u64(uint64_t v, uint64_t* red) {
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  v = warp_max_u64(v);
-  if (lane == 0) red[warp] = v;
-  __syncthreads();
-  if (warp == 0) {
-    uint64_t x = lane < kSelWarps ? red[lane] : 0ull;
-    x = warp_max_u64(x);
-    if (lane == 0) red[kSelWarps] = x;
-  }
-  __syncthreads();
-  const uint64_t r = red[kSelWarps];
-  __syncthreads();  // red[] is reused by the next call
-  return r;
-}
-
-__device__ __forceinline__ bool is_candidate(const float* delta, const uint8_t* valid,
-                                             int64_t n_tokens, int64_t abs_t, float& s) {
-  if (abs_t < 0 || abs_t >= n_tokens) return false;
-  if (valid && valid[abs_t] == 0) return false;
-  s = delta[abs_t];
-  return !isnan(s);
-}
-
-__global__ void __launch_bounds__(kSelThreads)
-    select_spacing_kernel(const float* __restrict__ delta, const uint8_t* __restrict__ valid,
-                           int64_t n_tokens, const int64_t* __restrict__ root_offsets,
-                           int32_t n_roots, int32_t k, int32_t min_gap, int32_t gap_mode,
-                           int32_t lo, int32_t hi, int32_t* __restrict__ branch_pos,
-                           int32_t* __restrict__ n_selected, float* __restrict__ branch_delta) {
-  __shared__ uint64_t red[kSelWarps + 1];
-  __shared__ int64_t chosen[kMaxK];
-  __shared__ int n_chosen;
-
-  for (int r = blockIdx.x; r < n_roots; r += gridDim.x) {
-    const int64_t start = root_offsets[r];
-    const int64_t end = root_offsets[r + 1];
-    const int64_t T = end > start ? end - start : 0;
-    const int64_t w_lo = lo > 0 ? lo : 0;
-    const int64_t w_hi = hi <= 0 ? T : (hi < T ? hi : T);
-    if (threadIdx.x == 0) n_chosen = 0;
-    __syncthreads();
-
-    if (min_gap <= 0 || gap_mode == 1) {
-      // plain top-k (also the first stage of drop-lower)
-      uint64_t top[kMaxK];
-#pragma unroll
-      for (int j = 0; j < kMaxK; ++j) top[j] = 0ull;
-      for (int64_t t = w_lo + threadIdx.x; t < w_hi; t += kSelThreads) {
-        float s;
-        if (!is_candidate(delta, valid, n_tokens, start + t, s)) continue;
-        const uint64_t key = make_key(s, t);
-        if (key > top[kMaxK - 1]) {
-#pragma unroll
-          for (int j = kMaxK - 1; j > 0; --j)
-            top[j] = key > top[j - 1] ? top[j - 1] : (key > top[j] ? key : top[j]);
-          top[0] = key > top[0] ? key : top[0];
-        }
-      }
-      for (int j = 0; j < k; ++j) {
-        const uint64_t best = block_max_u64(top[0], red);
-        if (best == 0ull) break;
-        if (top[0] == best) {
-#pragma unroll
-          for (int i = 0; i < kMaxK - 1; ++i) top[i] = top[i + 1];
-          top[kMaxK - 1] = 0ull;
-        }
-        if (threadIdx.x == 0) chosen[n_chosen++] = key_pos(best);
-      }
-      __syncthreads();
-      if (min_gap > 0 && threadIdx.x == 0) {
-        // drop-lower: keep, in rank order, the points not too close to a kept one
-        int kept = 0;
-        for (int i = 0; i < n_chosen; ++i) {
-          bool close = false;
-          for (int j = 0; j < kept; ++j) {
-            const int64_t dd = chosen[i] - chosen[j];
-            if ((dd < 0 ? -dd : dd) < min_gap) close = true;
-          }
-          if (!close) chosen[kept++] = chosen[i];
-        }
-        n_chosen = kept;
-      }
-    } else {
-      // greedy spacing: each round takes the best point compatible with all
-      // points accepted so far
-      for (int j = 0; j < k; ++j) {
-        const int na = n_chosen;
-        uint64_t mine = 0ull;
-        for (int64_t t = w_lo + threadIdx.x; t < w_hi; t += kSelThreads) {
-          float s;
-          if (!is_candidate(delta, valid, n_tokens, start + t, s)) continue;
-          bool close = false;
-          for (int i = 0; i < na; ++i) {
-            const int64_t dd = t - chosen[i];
-            if ((dd < 0 ? -dd : dd) < min_gap) close = true;
-          }
-          if (close) continue;
-          const uint64_t key = make_key(s, t);
-          mine = key > mine ? key : mine;
-        }
-        const uint64_t best = block_max_u64(mine, red);
-        if (best == 0ull) break;
-        if (threadIdx.x == 0) {
-          chosen[n_chosen] = key_pos(best);
-          n_chosen = n_chosen + 1;
-        }
-        __syncthreads();
-      }
-    }
-    __syncthreads();
-    if (threadIdx.x < k) {
-      const int j = threadIdx.x;
-      const int n = n_chosen;
-      const int64_t o = static_cast<int64_t>(r) * k + j;
-      if (j < n) {
-        branch_pos[o] = static_cast<int32_t>(chosen[j]);
-        if (branch_delta) branch_delta[o] = delta[start + chosen[j]];
-      } else {
-        branch_pos[o] = -1;
-        if (branch_delta) branch_delta[o] = __int_as_float(0x7fc00000);
-      }
-      if (j == 0) n_selected[r] = n;
-    }
-    if (k == 0 && threadIdx.x == 0) n_selected[r] = 0;
-    __syncthreads();
-  }
 }
 
 // The warp's running top-k is distributed over its lanes: lane j < k holds
@@ -284,13 +147,36 @@ __device__ __forceinline__ void wtk_offer_key(WarpTopK& w, uint64_t key, int k, 
   w.tau_s = fmaxf(key_score(w.tau), w.floor);
 }
 
+// Which root positions may enter a list: any (plain top-k), or, for the
+// greedy spacing rule, only those at least min_gap away from every point
+// accepted so far (the accepted list is the same on every lane).
+struct AnyPos {
+  static constexpr bool kAll = true;
+  __device__ __forceinline__ bool ok(int32_t) const { return true; }
+};
+
+struct FarFromAccepted {
+  static constexpr bool kAll = false;
+  const int32_t* acc;   // the group's accepted root positions (shared memory)
+  int na;
+  int32_t gap;
+  __device__ __forceinline__ bool ok(int32_t t) const {
+    for (int i = 0; i < na; ++i) {
+      const int32_t dd = t - acc[i];
+      if ((dd < 0 ? -dd : dd) < gap) return false;
+    }
+    return true;
+  }
+};
+
 // Offer each lane's candidate (score s at root position t; ok = valid): a
 // candidate whose score is below the k-th best's cannot beat it and is
 // rejected by the float compare alone; the others get their key built (NaN
 // scores never pass the compare).
+template <class F>
 __device__ __forceinline__ void wtk_offer(WarpTopK& w, float s, bool ok, int64_t t, int k,
-                                          int lane) {
-  ok = ok && s >= w.tau_s;
+                                          int lane, const F& f) {
+  ok = ok && s >= w.tau_s && f.ok(static_cast<int32_t>(t));
   if (!__any_sync(0xffffffffu, ok)) return;
   wtk_offer_key(w, ok ? make_key(s, t) : 0ull, k, lane);
 }
@@ -329,8 +215,9 @@ __device__ __forceinline__ void load_batch(Batch& b, const float* delta, const u
 // and one vote: no score reaches the threshold, so nothing can enter.
 // Otherwise the lanes' passing valid candidates are offered in rounds, each
 // lane its next one per round, until no lane has any left.
+template <class F>
 __device__ __forceinline__ void offer_batch(WarpTopK& w, const Batch& b, int32_t q,
-                                            int32_t start, int k, int lane) {
+                                            int32_t start, int k, int lane, const F& f) {
   float mx = -INFINITY;   // fmaxf ignores NaN scores
 #pragma unroll
   for (int i = 0; i < kBatch; ++i)
@@ -358,7 +245,7 @@ __device__ __forceinline__ void offer_batch(WarpTopK& w, const Batch& b, int32_t
       sj = j == 4 * i + 3 ? b.d[i].w : sj;
     }
     const int32_t t = q + 4 * (32 * (j >> 2) + lane) + (j & 3) - start;
-    wtk_offer_key(w, j >= 0 && sj >= w.tau_s ? make_key(sj, t) : 0ull, k, lane);
+    wtk_offer_key(w, j >= 0 && sj >= w.tau_s && f.ok(t) ? make_key(sj, t) : 0ull, k, lane);
   }
 }
 
@@ -381,14 +268,35 @@ __device__ __forceinline__ float warp_sort_desc_f(float x, int lane) {
 // among the k best of the slice.  Candidates below it are then rejected by
 // the float compare alone, which spares most of the insertions a root
 // otherwise pays while its list fills.
-__device__ __forceinline__ void set_floor(WarpTopK& w, const Batch& b, int k, int lane) {
+// Under a position filter a lane contributes its best valid candidate only
+// if the filter admits it (else -inf): the k-th largest contribution is
+// still reached by k distinct admitted candidates.
+template <class F>
+__device__ __forceinline__ void set_floor(WarpTopK& w, const Batch& b, int32_t q, int32_t start,
+                                          int k, int lane, const F& f) {
   float m = -INFINITY;   // fmaxf ignores a NaN operand
+  if constexpr (F::kAll) {
 #pragma unroll
-  for (int i = 0; i < kBatch; ++i) {
-    m = fmaxf(m, (b.v[i] & 0xFFu) != 0 ? b.d[i].x : -INFINITY);
-    m = fmaxf(m, (b.v[i] & 0xFF00u) != 0 ? b.d[i].y : -INFINITY);
-    m = fmaxf(m, (b.v[i] & 0xFF0000u) != 0 ? b.d[i].z : -INFINITY);
-    m = fmaxf(m, (b.v[i] & 0xFF000000u) != 0 ? b.d[i].w : -INFINITY);
+    for (int i = 0; i < kBatch; ++i) {
+      m = fmaxf(m, (b.v[i] & 0xFFu) != 0 ? b.d[i].x : -INFINITY);
+      m = fmaxf(m, (b.v[i] & 0xFF00u) != 0 ? b.d[i].y : -INFINITY);
+      m = fmaxf(m, (b.v[i] & 0xFF0000u) != 0 ? b.d[i].z : -INFINITY);
+      m = fmaxf(m, (b.v[i] & 0xFF000000u) != 0 ? b.d[i].w : -INFINITY);
+    }
+  } else {
+    int32_t at = 0;   // position of the lane's best (NaN never compares greater)
+#pragma unroll
+    for (int i = 0; i < kBatch; ++i) {
+      const int32_t t = q + 4 * (32 * i + lane) - start;
+      const float c[4] = {b.d[i].x, b.d[i].y, b.d[i].z, b.d[i].w};
+#pragma unroll
+      for (int j = 0; j < 4; ++j)
+        if (((b.v[i] >> (8 * j)) & 0xFFu) != 0 && c[j] > m) {
+          m = c[j];
+          at = t + j;
+        }
+    }
+    if (!f.ok(at)) m = -INFINITY;
   }
   m = warp_sort_desc_f(m, lane);
   w.floor = fmaxf(w.floor, __shfl_sync(0xffffffffu, m, k - 1));
@@ -399,10 +307,10 @@ __device__ __forceinline__ void set_floor(WarpTopK& w, const Batch& b, int k, in
 // `start`: a vector body walked in warp-uniform batches (all loads of a
 // batch issued before any is used; the first batch sets the floor), then the
 // scalar head and tail.
-template <bool kVec>
+template <bool kVec, class F>
 __device__ __forceinline__ void stream_range(WarpTopK& w, const float* delta, const uint8_t* valid,
                                              int64_t start64, int64_t a0_64, int64_t a1_64, int k,
-                                             int lane) {
+                                             int lane, const F& f) {
   const int32_t start = static_cast<int32_t>(start64);
   const int32_t a0 = static_cast<int32_t>(a0_64), a1 = static_cast<int32_t>(a1_64);
   if (!kVec) {
@@ -410,7 +318,7 @@ __device__ __forceinline__ void stream_range(WarpTopK& w, const float* delta, co
       const int32_t p = q + lane;
       const bool in = p < a1;
       wtk_offer(w, in ? delta[p] : 0.f, in && (valid == nullptr || valid[p] != 0), p - start, k,
-                lane);
+                lane, f);
     }
     return;
   }
@@ -422,21 +330,45 @@ __device__ __forceinline__ void stream_range(WarpTopK& w, const float* delta, co
       load_batch<true>(x, delta, valid, q, body, lane);
     else
       load_batch<false>(x, delta, valid, q, body, lane);
-    if (q == h) set_floor(w, x, k, lane);
-    offer_batch(w, x, q, start, k, lane);
+    if (q == h) set_floor(w, x, q, start, k, lane, f);
+    offer_batch(w, x, q, start, k, lane, f);
   }
   // scalar head and tail (at most 3 positions each)
   const int32_t p = lane < 4 ? a0 + lane : body + (lane - 4);
   const bool in = lane < 4 ? p < h : p < a1;
   wtk_offer(w, in ? delta[p] : 0.f, in && (valid == nullptr || valid[p] != 0), p - start, k,
-            lane);
+            lane, f);
 }
 
-// S warps share a root (S = 1, 2, 4, 8 in blocks of 8 warps, so 8/S roots
-// at a time per block; S = 16 in blocks of 16 warps): each warp streams one
-// contiguous slice of the root, then the group merges its S lists pairwise
-// through shared memory (a bitonic merge per level, the group's own named
-// barrier between levels) and its first warp writes the result.
+// Drop-lower spacing on a finished list (lanes 0..n-1, best first): in rank
+// order, a point within min_gap of a kept higher-ranked point is dropped;
+// the kept ones are packed to the front in rank order and n becomes their
+// count.
+__device__ __forceinline__ void drop_close(WarpTopK& w, int& n, int32_t min_gap, int lane) {
+  const int32_t t_me = static_cast<int32_t>(key_pos(w.mine));
+  bool keep = lane < n;
+  for (int i = 1; i < n; ++i) {
+    const int32_t t_i = __shfl_sync(0xffffffffu, t_me, i);
+    const int32_t dd = t_me - t_i;
+    const bool close = keep && lane < i && (dd < 0 ? -dd : dd) < min_gap;
+    if (__any_sync(0xffffffffu, close) && lane == i) keep = false;
+  }
+  const unsigned kept = __ballot_sync(0xffffffffu, keep);
+  uint64_t out = 0ull;
+  int j = 0;
+  for (int i = 0; i < n; ++i) {
+    const uint64_t ki = __shfl_sync(0xffffffffu, w.mine, i);
+    if ((kept >> i) & 1u) {
+      if (lane == j) out = ki;
+      ++j;
+    }
+  }
+  w.mine = out;
+  n = j;
+}
+
+// S warps share a root: S = 1, 2, 4, 8 in blocks of 8 warps (8/S roots at a
+// time per block), S = 16 in blocks of 16 warps.
 template <int S>
 struct TopkShape {
   static constexpr int kWarps = S == 16 ? 16 : 8;    // warps per block
@@ -448,17 +380,65 @@ __device__ __forceinline__ void group_sync(int id, int threads) {
   asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(threads) : "memory");
 }
 
-template <int S, bool kVec>
+// One pass of a root's group of S warps: every warp streams its slice of
+// [a0, a1) into a list of kk entries (positions the filter admits only),
+// then, for S > 1, the lists are merged pairwise into the first warp's
+// through shared memory (a bitonic merge per level, the group's own named
+// barrier between levels).  Returns true on the warp that holds the result.
+template <int S, bool kVec, class F>
+__device__ __forceinline__ bool collect(WarpTopK& w, uint64_t (*lists)[32], const float* delta,
+                                        const uint8_t* valid, int64_t start, int64_t a0,
+                                        int64_t a1, int kk, int lane, int warp, int grp, int ws,
+                                        const F& f) {
+  w = WarpTopK{0ull, 0ull, -INFINITY, -INFINITY};
+  if constexpr (S == 1) {
+    if (a1 > a0) stream_range<kVec>(w, delta, valid, start, a0, a1, kk, lane, f);
+    return true;
+  } else {
+    const int64_t len = a1 > a0 ? a1 - a0 : 0;
+    const int64_t per = ((len + S - 1) / S + 3) & ~int64_t{3};
+    const int64_t s0 = a0 + per * ws;
+    const int64_t s1 = s0 + per < a1 ? s0 + per : a1;
+    if (s0 < s1) stream_range<kVec>(w, delta, valid, start, s0, s1, kk, lane, f);
+    lists[warp][lane] = w.mine;
+    const int bar = 1 + grp, nthreads = 32 * S;
+    group_sync(bar, nthreads);
+#pragma unroll
+    for (int half = S / 2; half >= 1; half >>= 1) {
+      if (ws < half) {
+        const uint64_t m =
+            bitonic_merge16(lists[warp][lane & 15], lists[warp + half][(31 - lane) & 15], lane);
+        w.mine = lane < kk ? m : 0ull;
+        lists[warp][lane] = w.mine;
+      }
+      group_sync(bar, nthreads);
+    }
+    return ws == 0;
+  }
+}
+
+enum SelectMode : int { kPlain = 0, kDropLower = 1, kGreedy = 2 };
+
+// kMode: plain top-k; drop-lower spacing applied to the finished list; or
+// greedy spacing -- passes that each collect the kMaxK best positions far
+// enough from every point accepted so far and walk them in rank order,
+// accepting those still far enough, until k are accepted or a pass comes
+// back short (no candidate left).  Every pass but the last accepts at least
+// its first entry, so there are at most k passes; usually one to three.
+template <int S, bool kVec, int kMode>
 __global__ void __launch_bounds__(32 * TopkShape<S>::kWarps, TopkShape<S>::kMinBlocks)
     select_topk_kernel(const float* __restrict__ delta, const uint8_t* __restrict__ valid,
                        int64_t n_tokens, const int64_t* __restrict__ root_offsets,
-                       int32_t n_roots, int32_t k, int32_t lo, int32_t hi,
+                       int32_t n_roots, int32_t k, int32_t lo, int32_t hi, int32_t min_gap,
                        int32_t* __restrict__ branch_pos, int32_t* __restrict__ n_selected,
                        float* __restrict__ branch_delta) {
   using Sh = TopkShape<S>;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int grp = warp / S, ws = warp % S;
   __shared__ uint64_t lists[S == 1 ? 1 : Sh::kWarps][32];
+  // greedy: the group's accepted positions, then their count and whether
+  // the root is done (written by the warp that walks each pass's list)
+  __shared__ int32_t accepted[kMode == kGreedy ? Sh::kGroups : 1][kMaxK + 2];
   const int64_t step = static_cast<int64_t>(gridDim.x) * Sh::kGroups;
   for (int64_t r = static_cast<int64_t>(blockIdx.x) * Sh::kGroups + grp; r < n_roots; r += step) {
     const int64_t start = root_offsets[r];
@@ -469,43 +449,75 @@ __global__ void __launch_bounds__(32 * TopkShape<S>::kWarps, TopkShape<S>::kMinB
     int64_t a0 = start + w_lo, a1 = start + w_hi;
     if (a0 < 0) a0 = 0;
     if (a1 > n_tokens) a1 = n_tokens;
-    WarpTopK w{0ull, 0ull, -INFINITY, -INFINITY};
-    if constexpr (S == 1) {
-      if (a1 > a0) stream_range<kVec>(w, delta, valid, start, a0, a1, k, lane);
-    } else {
-      const int64_t len = a1 > a0 ? a1 - a0 : 0;
-      const int64_t per = ((len + S - 1) / S + 3) & ~int64_t{3};
-      const int64_t s0 = a0 + per * ws;
-      const int64_t s1 = s0 + per < a1 ? s0 + per : a1;
-      if (s0 < s1) stream_range<kVec>(w, delta, valid, start, s0, s1, k, lane);
-      lists[warp][lane] = w.mine;
-      const int bar = 1 + grp, nthreads = 32 * S;
-      group_sync(bar, nthreads);
-#pragma unroll
-      for (int half = S / 2; half >= 1; half >>= 1) {
-        if (ws < half) {
-          const uint64_t m =
-              bitonic_merge16(lists[warp][lane & 15], lists[warp + half][(31 - lane) & 15], lane);
-          w.mine = lane < k ? m : 0ull;
-          lists[warp][lane] = w.mine;
+    WarpTopK w;
+    if constexpr (kMode != kGreedy) {
+      if (!collect<S, kVec>(w, lists, delta, valid, start, a0, a1, k, lane, warp, grp, ws,
+                            AnyPos{}))
+        continue;
+      int n = __popc(__ballot_sync(0xffffffffu, w.mine != 0ull));
+      if constexpr (kMode == kDropLower) {
+        if (n > 1) drop_close(w, n, min_gap, lane);
+      }
+      if (lane < k) {
+        const int64_t o = r * k + lane;
+        if (lane < n) {
+          const int64_t t = key_pos(w.mine);
+          branch_pos[o] = static_cast<int32_t>(t);
+          // the key holds the absolute position minus the root start, mod 2^32
+          if (branch_delta)
+            branch_delta[o] = delta[static_cast<uint32_t>(start) + static_cast<uint32_t>(t)];
+        } else {
+          branch_pos[o] = -1;
+          if (branch_delta) branch_delta[o] = __int_as_float(0x7fc00000);
         }
-        group_sync(bar, nthreads);
       }
-      if (ws != 0) continue;
-    }
-    const int n = __popc(__ballot_sync(0xffffffffu, w.mine != 0ull));
-    if (lane < k) {
-      const int64_t o = r * k + lane;
-      if (lane < n) {
-        const int64_t t = key_pos(w.mine);
-        branch_pos[o] = static_cast<int32_t>(t);
-        if (branch_delta) branch_delta[o] = delta[start + t];
-      } else {
-        branch_pos[o] = -1;
-        if (branch_delta) branch_delta[o] = __int_as_float(0x7fc00000);
+      if (lane == 0) n_selected[r] = n;
+    } else {
+      int32_t* acc = accepted[grp];
+      FarFromAccepted far{acc, 0, min_gap};
+      bool holder = false;
+      for (;;) {
+        holder = collect<S, kVec>(w, lists, delta, valid, start, a0, a1, kMaxK, lane, warp, grp,
+                                  ws, far);
+        bool done = false;
+        if (holder) {
+          // every entry is far enough from the points accepted before this
+          // pass, so walking them in rank order is the drop-lower rule on
+          // the list: keep those not too close to a kept better one, and
+          // accept the first ones kept until k are accepted
+          const int m = __popc(__ballot_sync(0xffffffffu, w.mine != 0ull));
+          int kept = m;
+          if (kept > 1) drop_close(w, kept, min_gap, lane);
+          const int take = kept < k - far.na ? kept : k - far.na;
+          if (lane < take) acc[far.na + lane] = static_cast<int32_t>(key_pos(w.mine));
+          far.na += take;
+          done = far.na >= k || m < kMaxK;
+          if (lane == 0) {
+            acc[kMaxK] = far.na;
+            acc[kMaxK + 1] = done;
+          }
+        }
+        if constexpr (S > 1) {
+          group_sync(1 + grp, 32 * S);
+          far.na = acc[kMaxK];
+          done = acc[kMaxK + 1] != 0;
+        } else {
+          __syncwarp();
+        }
+        if (done) break;
       }
+      if (!holder) continue;
+      if (lane < k) {
+        const int64_t o = r * k + lane;
+        const bool have = lane < far.na;
+        const int32_t pos = have ? acc[lane] : -1;
+        branch_pos[o] = pos;
+        if (branch_delta)
+          branch_delta[o] = have ? delta[static_cast<uint32_t>(start) + static_cast<uint32_t>(pos)]
+                                 : __int_as_float(0x7fc00000);
+      }
+      if (lane == 0) n_selected[r] = far.na;
     }
-    if (lane == 0) n_selected[r] = n;
   }
 }
 
@@ -521,12 +533,22 @@ int select_split_override() {
   return v;
 }
 
-template <int S, bool kVec>
-hdl_status launch_topk_s(const float* delta, const uint8_t* valid, int64_t n_tokens,
-                         const int64_t* offs, int32_t n_roots, int32_t k, int32_t lo, int32_t hi,
-                         int32_t* bp, int32_t* ns, float* bd, int grid, cudaStream_t st) {
-  select_topk_kernel<S, kVec><<<grid, 32 * TopkShape<S>::kWarps, 0, st>>>(
-      delta, valid, n_tokens, offs, n_roots, k, lo, hi, bp, ns, bd);
+// Arguments of one selection launch (the kernel parameters after the grid).
+struct SelectArgs {
+  const float* delta;
+  const uint8_t* valid;
+  int64_t n_tokens;
+  const int64_t* offs;
+  int32_t n_roots, k, lo, hi, gap;
+  int32_t* bp;
+  int32_t* ns;
+  float* bd;
+};
+
+template <int S, bool kVec, int kMode>
+hdl_status launch_topk_s(const SelectArgs& a, int grid, cudaStream_t st) {
+  select_topk_kernel<S, kVec, kMode><<<grid, 32 * TopkShape<S>::kWarps, 0, st>>>(
+      a.delta, a.valid, a.n_tokens, a.offs, a.n_roots, a.k, a.lo, a.hi, a.gap, a.bp, a.ns, a.bd);
   return launch_status();
 }
 
@@ -539,41 +561,30 @@ hdl_status launch_topk_s(const float* delta, const uint8_t* valid, int64_t n_tok
 // took 47, 51, 67 and 84 us at S = 1, 2, 4, 8.  At S = 1 the kernel runs
 // within 8% of a read-only kernel with the same one-warp-per-root pattern
 // and occupancy; neither deeper register prefetch nor a shared-memory ring
-// filled by bulk copies made it faster.)
-template <bool kVec>
-hdl_status launch_topk(const float* delta, const uint8_t* valid, int64_t n_tokens,
-                       const int64_t* offs, int32_t n_roots, int32_t k, int32_t lo, int32_t hi,
-                       int32_t* bp, int32_t* ns, float* bd, int sms, cudaStream_t st) {
-  if (n_roots < 2 * sms)
-    return launch_topk_s<16, kVec>(delta, valid, n_tokens, offs, n_roots, k, lo, hi, bp, ns, bd,
-                                   n_roots, st);
+// filled by bulk copies made it faster.)  kMode selects the spacing rule,
+// with min_gap = a.gap.
+template <bool kVec, int kMode>
+hdl_status launch_topk(const SelectArgs& a, int sms, cudaStream_t st) {
+  if (a.n_roots < 2 * sms) return launch_topk_s<16, kVec, kMode>(a, a.n_roots, st);
   int per_sm = 0;
-  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, select_topk_kernel<1, kVec>, 256,
-                                                    0) != cudaSuccess || per_sm <= 0)
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, select_topk_kernel<1, kVec, kMode>,
+                                                    256, 0) != cudaSuccess || per_sm <= 0)
     per_sm = 4;
   const int64_t resident_warps = static_cast<int64_t>(per_sm) * 8 * sms;
-  int64_t span = n_tokens / n_roots;
-  if (hi > 0 && hi < span) span = hi;
-  span -= lo > 0 ? lo : 0;
+  int64_t span = a.n_tokens / a.n_roots;
+  if (a.hi > 0 && a.hi < span) span = a.hi;
+  span -= a.lo > 0 ? a.lo : 0;
   int S = 1;
-  while (S < 8 && int64_t{n_roots} * S < resident_warps && span / (2 * S) >= 1024) S *= 2;
+  while (S < 8 && int64_t{a.n_roots} * S < resident_warps && span / (2 * S) >= 1024) S *= 2;
   if (const int forced = select_split_override()) S = forced;
-  const int64_t blocks = (int64_t{n_roots} * S + 7) / 8;
+  const int64_t blocks = (int64_t{a.n_roots} * S + 7) / 8;
   const int64_t cap = static_cast<int64_t>(per_sm) * sms;
   const int grid = static_cast<int>(blocks < cap ? blocks : cap);
   switch (S) {
-    case 1:
-      return launch_topk_s<1, kVec>(delta, valid, n_tokens, offs, n_roots, k, lo, hi, bp, ns, bd,
-                                    grid, st);
-    case 2:
-      return launch_topk_s<2, kVec>(delta, valid, n_tokens, offs, n_roots, k, lo, hi, bp, ns, bd,
-                                    grid, st);
-    case 4:
-      return launch_topk_s<4, kVec>(delta, valid, n_tokens, offs, n_roots, k, lo, hi, bp, ns, bd,
-                                    grid, st);
-    default:
-      return launch_topk_s<8, kVec>(delta, valid, n_tokens, offs, n_roots, k, lo, hi, bp, ns, bd,
-                                    grid, st);
+    case 1: return launch_topk_s<1, kVec, kMode>(a, grid, st);
+    case 2: return launch_topk_s<2, kVec, kMode>(a, grid, st);
+    case 4: return launch_topk_s<4, kVec, kMode>(a, grid, st);
+    default: return launch_topk_s<8, kVec, kMode>(a, grid, st);
   }
 }
 
@@ -605,21 +616,18 @@ extern "C" hdl_status hdl_select_branches(const float* delta, const uint8_t* val
   const int sms = current_sm_count();
   if (sms <= 0) return HDL_ERR_CUDA;
   cudaStream_t st = as_stream(cuda_stream);
-  if (o.min_gap > 0) {
-    const int grid = n_roots < 32 * sms ? n_roots : 32 * sms;
-    select_spacing_kernel<<<grid, kSelThreads, 0, st>>>(
-        delta, valid, n_tokens, root_offsets, n_roots, k, o.min_gap, o.gap_mode, o.lo, o.hi,
-        branch_pos, n_selected, branch_delta);
-    return launch_status();
-  }
   if (k == 0) {
     if (cudaMemsetAsync(n_selected, 0, sizeof(int32_t) * n_roots, st) != cudaSuccess)
       return HDL_ERR_CUDA;
     return HDL_OK;
   }
   const bool vec = aligned_to(delta, 16) && (valid == nullptr || aligned_to(valid, 4));
-  return vec ? launch_topk<true>(delta, valid, n_tokens, root_offsets, n_roots, k, o.lo, o.hi,
-                                 branch_pos, n_selected, branch_delta, sms, st)
-             : launch_topk<false>(delta, valid, n_tokens, root_offsets, n_roots, k, o.lo, o.hi,
-                                  branch_pos, n_selected, branch_delta, sms, st);
+  const SelectArgs a{delta, valid, n_tokens, root_offsets, n_roots, k, o.lo, o.hi, o.min_gap,
+                     branch_pos, n_selected, branch_delta};
+  if (o.min_gap > 0 && o.gap_mode == 0)
+    return vec ? launch_topk<true, kGreedy>(a, sms, st) : launch_topk<false, kGreedy>(a, sms, st);
+  if (o.min_gap > 0)
+    return vec ? launch_topk<true, kDropLower>(a, sms, st)
+               : launch_topk<false, kDropLower>(a, sms, st);
+  return vec ? launch_topk<true, kPlain>(a, sms, st) : launch_topk<false, kPlain>(a, sms, st);
 }

@@ -89,6 +89,65 @@ def test_select_window(hdl):
         assert_select_equal(hdl, delta, valid, offs, 8, lo=lo, hi=hi)
 
 
+def add_spikes(delta, offs, seed, spans=3, width=32, lift=5.0):
+    """Clustered high scores (the shape divergence takes around a decisive
+    token): `spans` runs of `width` positions per root lifted by `lift`."""
+    rng = np.random.default_rng(seed)
+    for r in range(len(offs) - 1):
+        T = int(offs[r + 1] - offs[r])
+        for _ in range(spans if T > width else 0):
+            a = int(offs[r]) + int(rng.integers(0, T - width))
+            delta[a:a + width] += lift
+    return delta
+
+
+@pytest.mark.parametrize("gap_mode", [0, 1])
+def test_select_spacing_many_roots(hdl, gap_mode):
+    """The spacing rule with many roots (one warp per root; greedy keeps a
+    per-thread list and rescans only when it runs dry), clustered scores so
+    that whole runs are ruled out at once, gaps from 1 (plain top-k) to longer
+    than the roots, windows, ties, NaN and +-inf: bit-exact against the
+    oracle."""
+    rng = np.random.default_rng(40 + gap_mode)
+    lengths = list(rng.integers(0, 2000, size=400)) + [0, 1, 2, 3, 4, 5, 40, 70000]
+    for seed, ties in ((0, None), (1, 4)):
+        delta, valid, offs = make_roots(lengths, 50 + seed, tie_levels=ties, nan_frac=0.01)
+        delta = add_spikes(delta, offs, seed)
+        delta[::997] = np.inf
+        delta[5::1013] = -np.inf
+        for k in (1, 8, 16):
+            for min_gap in (1, 3, 40, 5000):
+                assert_select_equal(hdl, delta, valid, offs, k, min_gap=min_gap,
+                                    gap_mode=gap_mode)
+        for lo, hi in ((10, 0), (100, 900)):
+            assert_select_equal(hdl, delta, None, offs, 8, min_gap=20, gap_mode=gap_mode,
+                                lo=lo, hi=hi)
+
+
+@pytest.mark.parametrize("n_roots", [7, 500])
+@pytest.mark.parametrize("gap_mode", [0, 1])
+def test_select_spacing_unaligned(hdl, n_roots, gap_mode):
+    """Scores / validity off their 16- / 4-byte alignment: the scalar paths
+    of both spacing modes, with few and with many roots."""
+    lengths = list(np.random.default_rng(n_roots).integers(0, 2500, size=n_roots))
+    delta, valid, offs = make_roots(lengths, 13, tie_levels=6)
+    delta = add_spikes(delta, offs, 3)
+    N = len(delta)
+    d = torch.zeros(N + 1, dtype=torch.float32, device="cuda")
+    v = torch.zeros(N + 1, dtype=torch.uint8, device="cuda")
+    d[1:] = torch.from_numpy(delta).cuda()
+    v[1:] = torch.from_numpy(valid).cuda()
+    o = torch.from_numpy(offs).cuda()
+    for min_gap in (2, 33):
+        bp, ns, bd = hdl.hdl_select_branches(d[1:], v[1:], o, 16, min_gap=min_gap,
+                                             gap_mode=gap_mode)
+        pos, nsel, val = oracle.select_branches(delta.astype(np.float64), valid, offs, 16,
+                                                min_gap=min_gap, gap_mode=gap_mode)
+        assert np.array_equal(ns.cpu().numpy(), nsel)
+        assert np.array_equal(bp.cpu().numpy(), pos)
+        assert np.array_equal(bd.cpu().numpy().astype(np.float64), val, equal_nan=True)
+
+
 @pytest.mark.parametrize("gap_mode", [0, 1])
 @pytest.mark.parametrize("min_gap", [1, 2, 7, 64])
 def test_select_spacing(hdl, gap_mode, min_gap):
@@ -225,6 +284,8 @@ for k in (1, 8, 16):
         out[f"bp{k}_{lo}"] = bp.cpu().numpy()
         out[f"ns{k}_{lo}"] = ns.cpu().numpy()
         out[f"bd{k}_{lo}"] = bd.cpu().numpy()
+    bp, ns, bd = hdl.hdl_select_branches(d, v, o, k, min_gap=6, gap_mode=1)
+    out[f"bp{k}_drop"], out[f"ns{k}_drop"] = bp.cpu().numpy(), ns.cpu().numpy()
 np.savez(sys.argv[3], **out)
 """
 
@@ -251,6 +312,10 @@ def test_select_warps_per_root(hdl, tmp_path, split):
             assert np.array_equal(got[f"ns{k}_{lo}"], nsel)
             assert np.array_equal(got[f"bp{k}_{lo}"], pos)
             assert np.array_equal(got[f"bd{k}_{lo}"].astype(np.float64), val, equal_nan=True)
+        pos, nsel, _ = oracle.select_branches(delta.astype(np.float64), valid, offs, k,
+                                              min_gap=6, gap_mode=1)
+        assert np.array_equal(got[f"ns{k}_drop"], nsel)
+        assert np.array_equal(got[f"bp{k}_drop"], pos)
 
 
 def test_select_randomized(hdl):
