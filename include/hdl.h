@@ -204,7 +204,10 @@ HDL_API hdl_status hdl_merge_vocab_shards(const float* stats, int32_t n_shards,
  *   stats           [4] float out: loss, masked tokens, fraction of masked
  *                   tokens whose clipped term is strictly smaller, mean ratio.
  *   workspace       hdl_grpo_loss_workspace_bytes() bytes, 256-byte aligned.
- * The loss is reduced in double precision in a fixed order. */
+ * The loss is reduced in double precision in a fixed order.  Every array is
+ * aligned to its element type; the token streams are read 16 bytes at a time
+ * when the addresses of logp_new, logp_old and grad (/ 4) and of mask agree
+ * mod 4, else one token at a time (same results). */
 HDL_API size_t hdl_grpo_loss_workspace_bytes(void);
 
 HDL_API hdl_status hdl_grpo_loss(const float* logp_new, const float* logp_old,
@@ -296,7 +299,11 @@ typedef struct {
  *                  order, -1 after the last selected one.
  *   n_selected     [n_roots] int32 out: number of points selected (<= k).
  *   branch_delta   [n_roots * k] float out or NULL: delta at each point, NaN
- *                  padding. */
+ *                  padding.
+ * Every array is aligned to its element type.  The scores are read 16 bytes
+ * at a time when delta's address / 4 and valid's address agree mod 4 (both
+ * from the same token offset of aligned buffers, for instance), else one
+ * element at a time (same results). */
 HDL_API hdl_status hdl_select_branches(const float* delta, const uint8_t* valid,
                                int64_t n_tokens, const int64_t* root_offsets,
                                int32_t n_roots, int32_t k,
@@ -339,6 +346,8 @@ HDL_API hdl_status hdl_assign_continuations(const int32_t* n_selected,
  *   cont_valid    [mask_len] uint8, same packing as mask, or NULL.
  *   mask          [mask_len] uint8 out; bytes outside
  *                 [cont_offsets[0], cont_offsets[n_cont]) are left untouched.
+ * 16-byte vectors are used when mask and cont_valid have the same address
+ * mod 16, else single bytes (same results).
  */
 HDL_API hdl_status hdl_suffix_mask(const int32_t* cont_branch,
                            const int64_t* cont_offsets, int32_t n_cont,

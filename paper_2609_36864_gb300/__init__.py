@@ -159,6 +159,17 @@ def _dev(t: torch.Tensor, name: str, dtype=None, numel: Optional[int] = None,
         raise ValueError(f"{name} must hold {numel} elements (got {t.numel()})")
 
 
+def _empty_like_phase(n: int, dtype, like: torch.Tensor, period: int) -> torch.Tensor:
+    """An empty [n] tensor whose address has the same residue mod `period`
+    bytes as `like`'s, so that the kernels' 16-byte vector paths (taken when
+    the streams' alignments agree) still apply to sliced inputs."""
+    esize = torch.empty(0, dtype=dtype).element_size()
+    shift = (like.data_ptr() % period) // esize
+    buf = torch.empty(n + period // esize, dtype=dtype, device=like.device)
+    off = (shift - buf.data_ptr() % period // esize) % (period // esize)
+    return buf[off:off + n]
+
+
 def _lm_inputs(h_orig, h_hind, w, targets, w_name="w_lmhead"):
     """Validate the operands of a re-scoring call; returns (dtype code, N, d, V, device)."""
     _dev(h_orig, "h_orig")
@@ -361,7 +372,10 @@ def hdl_suffix_mask(cont_branch, cont_offsets, cont_valid=None, mask=None,
             mask_len = cont_valid.numel() if cont_valid is not None else None
         if mask_len is None:
             raise ValueError("give mask, mask_len or cont_valid")
-        mask = torch.zeros(mask_len, dtype=torch.uint8, device=dev)
+        if cont_valid is not None:
+            mask = _empty_like_phase(mask_len, torch.uint8, cont_valid, 16).zero_()
+        else:
+            mask = torch.zeros(mask_len, dtype=torch.uint8, device=dev)
     _dev(mask, "mask", torch.uint8, device=dev)
     if cont_valid is not None and cont_valid.numel() != mask.numel():
         raise ValueError("cont_valid and mask must have the same length")
@@ -471,7 +485,7 @@ def hdl_grpo_loss(logp_new, logp_old, mask, traj_offsets, rewards, group_offsets
     if advantages is None:
         advantages = torch.zeros(J, dtype=torch.float32, device=dev)
     if grad is None and want_grad:
-        grad = torch.empty(T, dtype=torch.float32, device=dev)
+        grad = _empty_like_phase(T, torch.float32, logp_new, 16)
     if stats is None:
         stats = torch.empty(4, dtype=torch.float32, device=dev)
     if workspace is None:

@@ -185,7 +185,7 @@ __global__ void __launch_bounds__(kThreads, 4)
                       const float* __restrict__ adv, float eps_low, float eps_high,
                       const unsigned long long* __restrict__ counts, int n_count_blocks,
                       float* __restrict__ grad, Sums* __restrict__ partial,
-                      unsigned int* __restrict__ done, float* __restrict__ stats) {
+                      unsigned int* __restrict__ done, float* __restrict__ stats, int32_t phase) {
   __shared__ float red[kThreads / 32][4];
   __shared__ double red_d[kThreads / 32][4];
   __shared__ float s_scale;
@@ -210,7 +210,8 @@ __global__ void __launch_bounds__(kThreads, 4)
   TokenOut acc{0.f, 0.f, 0.f};
   int ntok = 0;
   // tokens [s, e) of one trajectory, advantage A: head and tail one token
-  // per lane, the 16-byte-aligned body three 4-token groups per lane at a time
+  // per lane, the body three 4-token groups per lane at a time (groups start
+  // at tokens p with (p + phase) % 4 == 0, where every stream is aligned)
   auto stream_trajectory = [&](int64_t s, int64_t e, float A) {
     auto one = [&](int64_t u) {
       float g = 0.f;
@@ -222,7 +223,7 @@ __global__ void __launch_bounds__(kThreads, 4)
     };
     int64_t h = s, body = s;
     if (kVec) {
-      h = (s + 3) & ~int64_t{3};
+      h = ((s + phase + 3) & ~int64_t{3}) - phase;
       h = h < e ? h : e;
       body = h + ((e - h) & ~int64_t{3});
     }
@@ -354,7 +355,8 @@ extern "C" hdl_status hdl_grpo_loss(const float* logp_new, const float* logp_old
   if (n_traj > 0 && !traj_offsets) return HDL_ERR_INVALID_ARG;
   if (n_tokens > 0 && (!logp_new || !logp_old || !mask || n_traj == 0))
     return HDL_ERR_INVALID_ARG;
-  if (!aligned_to(stats, 4) || (advantages && !aligned_to(advantages, 4)) ||
+  if ((logp_new && !aligned_to(logp_new, 4)) || (logp_old && !aligned_to(logp_old, 4)) ||
+      !aligned_to(stats, 4) || (advantages && !aligned_to(advantages, 4)) ||
       (traj_offsets && !aligned_to(traj_offsets, 8)) ||
       (group_offsets && !aligned_to(group_offsets, 4)) || (grad && !aligned_to(grad, 4)))
     return HDL_ERR_INVALID_ARG;
@@ -369,8 +371,15 @@ extern "C" hdl_status hdl_grpo_loss(const float* logp_new, const float* logp_old
       static_cast<uint8_t*>(workspace) + align_up(kMaxBlocks * sizeof(Sums), 256));
   auto* done = reinterpret_cast<unsigned int*>(
       reinterpret_cast<uint8_t*>(counts) + align_up(kMaxBlocks * sizeof(unsigned long long), 256));
-  const bool vec = n_tokens > 0 && aligned_to(logp_new, 16) && aligned_to(logp_old, 16) &&
-                   aligned_to(mask, 4) && (grad == nullptr || aligned_to(grad, 16));
+  // 16-byte vectors wherever the four token streams' alignments agree
+  // (buffers sliced at the same token offset included)
+  const auto f_phase = [](const void* q) {
+    return static_cast<int>((reinterpret_cast<uintptr_t>(q) >> 2) & 3u);
+  };
+  const int phase = f_phase(logp_new);
+  const bool vec = n_tokens > 0 && f_phase(logp_old) == phase &&
+                   static_cast<int>(reinterpret_cast<uintptr_t>(mask) & 3u) == phase &&
+                   (grad == nullptr || f_phase(grad) == phase);
   // persistent grids: as many blocks as are resident at once (<= kMaxBlocks)
   int per_sm = 0;
   if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, grpo_token_kernel<true, false>,
@@ -403,6 +412,6 @@ extern "C" hdl_status hdl_grpo_loss(const float* logp_new, const float* logp_old
   if (launch_status() != HDL_OK) return HDL_ERR_CUDA;
   tok<<<blocks, kThreads, 0, st>>>(logp_new, logp_old, mask, n_tokens, traj_offsets, n_traj,
                                    advantages, eps_low, eps_high, counts, prep, grad, partial,
-                                   done, stats);
+                                   done, stats, phase);
   return launch_status();
 }

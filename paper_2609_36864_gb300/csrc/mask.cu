@@ -94,15 +94,17 @@ __device__ __forceinline__ uint32_t nonzero_bytes(uint32_t w) {
 
 // One warp per continuation c: bytes [s, e) = [offs[c], offs[c+1]) clipped to
 // the mask; byte p is on iff p >= thr (= s + b, or never when b < 0) and it is
-// valid.  The 16-byte-aligned body is read and written 16 bytes per lane, the
-// head and tail bytes one by one, and only the one vector that contains thr
-// is resolved byte by byte; four body vectors per lane are loaded before any
-// is stored (one at a time measured 5-8 % slower).
+// valid.  The body, whose vectors start at bytes p with (p + phase) % 16 == 0
+// (phase = the mask's address mod 16, the validity bytes' too), is read and
+// written 16 bytes per lane, the head and tail bytes one by one, and only the
+// one vector that contains thr is resolved byte by byte; four body vectors
+// per lane are loaded before any is stored (one at a time measured 5-8 %
+// slower).
 template <bool kVec>
 __global__ void __launch_bounds__(kMaskThreads)
     suffix_mask_kernel(const int32_t* __restrict__ cb, const int64_t* __restrict__ offs,
                        int32_t n_cont, const uint8_t* __restrict__ valid,
-                       uint8_t* __restrict__ mask, int64_t mask_len) {
+                       uint8_t* __restrict__ mask, int64_t mask_len, int32_t phase) {
   const int lane = threadIdx.x & 31;
   const int64_t warps = static_cast<int64_t>(gridDim.x) * (blockDim.x / 32);
   for (int64_t c = static_cast<int64_t>(blockIdx.x) * (blockDim.x / 32) + (threadIdx.x >> 5);
@@ -115,7 +117,7 @@ __global__ void __launch_bounds__(kMaskThreads)
     if (e <= s) continue;
     int64_t h = s, body = s;
     if (kVec) {
-      h = (s + 15) & ~int64_t{15};
+      h = ((s + phase + 15) & ~int64_t{15}) - phase;
       h = h < e ? h : e;
       body = h + ((e - h) & ~int64_t{15});
     }
@@ -190,7 +192,10 @@ extern "C" hdl_status hdl_suffix_mask(const int32_t* cont_branch, const int64_t*
   if (n_cont == 0 || mask_len == 0) return HDL_OK;
   if (!cont_branch || !cont_offsets || !mask) return HDL_ERR_INVALID_ARG;
   if (!aligned_to(cont_branch, 4) || !aligned_to(cont_offsets, 8)) return HDL_ERR_INVALID_ARG;
-  const bool vec = aligned_to(mask, 16) && (cont_valid == nullptr || aligned_to(cont_valid, 16));
+  // 16-byte vectors wherever the mask's and validity bytes' alignments agree
+  const int phase = static_cast<int>(reinterpret_cast<uintptr_t>(mask) & 15u);
+  const bool vec = cont_valid == nullptr ||
+                   static_cast<int>(reinterpret_cast<uintptr_t>(cont_valid) & 15u) == phase;
   const int sms = current_sm_count();
   if (sms <= 0) return HDL_ERR_CUDA;
   const int64_t blocks = ceil_div(n_cont, kMaskThreads / 32);   // one warp per continuation
@@ -198,9 +203,9 @@ extern "C" hdl_status hdl_suffix_mask(const int32_t* cont_branch, const int64_t*
   cudaStream_t st = as_stream(cuda_stream);
   if (vec)
     suffix_mask_kernel<true><<<grid, kMaskThreads, 0, st>>>(cont_branch, cont_offsets, n_cont,
-                                                            cont_valid, mask, mask_len);
+                                                            cont_valid, mask, mask_len, phase);
   else
     suffix_mask_kernel<false><<<grid, kMaskThreads, 0, st>>>(cont_branch, cont_offsets, n_cont,
-                                                             cont_valid, mask, mask_len);
+                                                             cont_valid, mask, mask_len, phase);
   return launch_status();
 }

@@ -310,7 +310,7 @@ __device__ __forceinline__ void set_floor(WarpTopK& w, const Batch& b, int32_t q
 template <bool kVec, class F>
 __device__ __forceinline__ void stream_range(WarpTopK& w, const float* delta, const uint8_t* valid,
                                              int64_t start64, int64_t a0_64, int64_t a1_64, int k,
-                                             int lane, const F& f) {
+                                             int lane, int phase, const F& f) {
   const int32_t start = static_cast<int32_t>(start64);
   const int32_t a0 = static_cast<int32_t>(a0_64), a1 = static_cast<int32_t>(a1_64);
   if (!kVec) {
@@ -322,7 +322,10 @@ __device__ __forceinline__ void stream_range(WarpTopK& w, const float* delta, co
     }
     return;
   }
-  const int32_t h = a0 + ((4 - (a0 & 3)) & 3) < a1 ? a0 + ((4 - (a0 & 3)) & 3) : a1;
+  // vector positions q have (q + phase) % 4 == 0: delta + q is 16-byte and
+  // valid + q 4-byte aligned
+  const int32_t up = a0 + ((4 - ((a0 + phase) & 3)) & 3);
+  const int32_t h = up < a1 ? up : a1;
   const int32_t body = h + ((a1 - h) & ~3);
   for (int32_t q = h; q < body; q += kSpan) {
     Batch x;
@@ -389,17 +392,17 @@ template <int S, bool kVec, class F>
 __device__ __forceinline__ bool collect(WarpTopK& w, uint64_t (*lists)[32], const float* delta,
                                         const uint8_t* valid, int64_t start, int64_t a0,
                                         int64_t a1, int kk, int lane, int warp, int grp, int ws,
-                                        const F& f) {
+                                        int phase, const F& f) {
   w = WarpTopK{0ull, 0ull, -INFINITY, -INFINITY};
   if constexpr (S == 1) {
-    if (a1 > a0) stream_range<kVec>(w, delta, valid, start, a0, a1, kk, lane, f);
+    if (a1 > a0) stream_range<kVec>(w, delta, valid, start, a0, a1, kk, lane, phase, f);
     return true;
   } else {
     const int64_t len = a1 > a0 ? a1 - a0 : 0;
     const int64_t per = ((len + S - 1) / S + 3) & ~int64_t{3};
     const int64_t s0 = a0 + per * ws;
     const int64_t s1 = s0 + per < a1 ? s0 + per : a1;
-    if (s0 < s1) stream_range<kVec>(w, delta, valid, start, s0, s1, kk, lane, f);
+    if (s0 < s1) stream_range<kVec>(w, delta, valid, start, s0, s1, kk, lane, phase, f);
     lists[warp][lane] = w.mine;
     const int bar = 1 + grp, nthreads = 32 * S;
     group_sync(bar, nthreads);
@@ -430,8 +433,8 @@ __global__ void __launch_bounds__(32 * TopkShape<S>::kWarps, TopkShape<S>::kMinB
     select_topk_kernel(const float* __restrict__ delta, const uint8_t* __restrict__ valid,
                        int64_t n_tokens, const int64_t* __restrict__ root_offsets,
                        int32_t n_roots, int32_t k, int32_t lo, int32_t hi, int32_t min_gap,
-                       int32_t* __restrict__ branch_pos, int32_t* __restrict__ n_selected,
-                       float* __restrict__ branch_delta) {
+                       int32_t phase, int32_t* __restrict__ branch_pos,
+                       int32_t* __restrict__ n_selected, float* __restrict__ branch_delta) {
   using Sh = TopkShape<S>;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int grp = warp / S, ws = warp % S;
@@ -451,7 +454,7 @@ __global__ void __launch_bounds__(32 * TopkShape<S>::kWarps, TopkShape<S>::kMinB
     if (a1 > n_tokens) a1 = n_tokens;
     WarpTopK w;
     if constexpr (kMode != kGreedy) {
-      if (!collect<S, kVec>(w, lists, delta, valid, start, a0, a1, k, lane, warp, grp, ws,
+      if (!collect<S, kVec>(w, lists, delta, valid, start, a0, a1, k, lane, warp, grp, ws, phase,
                             AnyPos{}))
         continue;
       int n = __popc(__ballot_sync(0xffffffffu, w.mine != 0ull));
@@ -478,7 +481,7 @@ __global__ void __launch_bounds__(32 * TopkShape<S>::kWarps, TopkShape<S>::kMinB
       bool holder = false;
       for (;;) {
         holder = collect<S, kVec>(w, lists, delta, valid, start, a0, a1, kMaxK, lane, warp, grp,
-                                  ws, far);
+                                  ws, phase, far);
         bool done = false;
         if (holder) {
           // every entry is far enough from the points accepted before this
@@ -540,6 +543,7 @@ struct SelectArgs {
   int64_t n_tokens;
   const int64_t* offs;
   int32_t n_roots, k, lo, hi, gap;
+  int32_t phase;   // (delta address / 4) mod 4; valid's address has the same residue mod 4
   int32_t* bp;
   int32_t* ns;
   float* bd;
@@ -548,7 +552,8 @@ struct SelectArgs {
 template <int S, bool kVec, int kMode>
 hdl_status launch_topk_s(const SelectArgs& a, int grid, cudaStream_t st) {
   select_topk_kernel<S, kVec, kMode><<<grid, 32 * TopkShape<S>::kWarps, 0, st>>>(
-      a.delta, a.valid, a.n_tokens, a.offs, a.n_roots, a.k, a.lo, a.hi, a.gap, a.bp, a.ns, a.bd);
+      a.delta, a.valid, a.n_tokens, a.offs, a.n_roots, a.k, a.lo, a.hi, a.gap, a.phase, a.bp,
+      a.ns, a.bd);
   return launch_status();
 }
 
@@ -621,9 +626,13 @@ extern "C" hdl_status hdl_select_branches(const float* delta, const uint8_t* val
       return HDL_ERR_CUDA;
     return HDL_OK;
   }
-  const bool vec = aligned_to(delta, 16) && (valid == nullptr || aligned_to(valid, 4));
+  // 16-byte vectors wherever the scores' and validity bytes' alignments agree
+  // (buffers sliced at the same token offset included)
+  const int phase = static_cast<int>((reinterpret_cast<uintptr_t>(delta) >> 2) & 3u);
+  const bool vec = valid == nullptr ||
+                   static_cast<int>(reinterpret_cast<uintptr_t>(valid) & 3u) == phase;
   const SelectArgs a{delta, valid, n_tokens, root_offsets, n_roots, k, o.lo, o.hi, o.min_gap,
-                     branch_pos, n_selected, branch_delta};
+                     phase, branch_pos, n_selected, branch_delta};
   if (o.min_gap > 0 && o.gap_mode == 0)
     return vec ? launch_topk<true, kGreedy>(a, sms, st) : launch_topk<false, kGreedy>(a, sms, st);
   if (o.min_gap > 0)

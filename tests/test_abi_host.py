@@ -183,3 +183,18 @@ def test_rescore_ex_options_and_workspace(L):
     small = hdl.hdl_rescore_workspace_bytes(16, 64, 100)
     assert L.hdl_rescore_ex(P, P, P, 0, P, 16, 64, 100, P, P, None, ctypes.byref(o), P,
                             small, None) == 3
+
+
+def test_binding_allocates_outputs_at_the_inputs_phase():
+    """Outputs the binding allocates (GRPO gradient, suffix mask) start at the
+    same address residue mod 16 as the input they stream with, so sliced
+    inputs keep the kernels' 16-byte vector paths."""
+    import torch
+    from paper_2609_36864_gb300 import _empty_like_phase
+    for dt in (torch.float32, torch.uint8):
+        es = torch.empty(0, dtype=dt).element_size()
+        for off in range(16 // es):
+            like = torch.empty(100 + off, dtype=dt)[off:]
+            out = _empty_like_phase(37, dt, like, 16)
+            assert out.numel() == 37 and out.dtype == dt
+            assert out.data_ptr() % 16 == like.data_ptr() % 16

@@ -96,15 +96,21 @@ def test_select_assign_mask_stay_in_bounds(hdl):
     lens = rng.integers(0, 300, size=C)
     coffs = torch.tensor(np.concatenate([[0], np.cumsum(lens)]), dtype=torch.int64, device="cuda")
     total = int(coffs[-1])
-    cv = (torch.rand(total, device="cuda") < 0.7).to(torch.uint8)
-    for offset in (0, 1):                         # vector and byte paths
+    cv_all = (torch.rand(total + 16, device="cuda") < 0.7).to(torch.uint8)
+    # (mask, validity) offsets from 16-byte alignment: vector path, byte path,
+    # phase-shifted vector path
+    for offset, v_off in ((0, 0), (1, 0), (3, 3)):
         m = Guarded((total,), torch.uint8, offset=offset)
+        cv = cv_all[v_off:v_off + total]
         hdl.hdl_suffix_mask(cb.t, coffs, cv, mask=m.t)
         torch.cuda.synchronize()
         assert m.intact()
 
 
-def test_grpo_stays_in_bounds(hdl):
+@pytest.mark.parametrize("phase", [0, 1, 3])
+def test_grpo_stays_in_bounds(hdl, phase):
+    """Token streams `phase` elements off 16-byte alignment (all four alike:
+    the vector path, shifted when phase > 0)."""
     rng = np.random.default_rng(4)
     sizes = rng.integers(1, 17, size=50)
     goffs = torch.tensor(np.concatenate([[0], np.cumsum(sizes)]), dtype=torch.int32,
@@ -114,12 +120,13 @@ def test_grpo_stays_in_bounds(hdl):
     toffs = torch.tensor(np.concatenate([[0], np.cumsum(lens)]), dtype=torch.int64,
                          device="cuda")
     T = int(toffs[-1])
-    lpo = -torch.rand(T, device="cuda")
-    lpn = lpo + 0.3 * torch.randn(T, device="cuda")
-    m = (torch.rand(T, device="cuda") < 0.7).to(torch.uint8)
+    lpo = -torch.rand(T + phase, device="cuda")[phase:]
+    lpn = (lpo + 0.3 * torch.randn(T, device="cuda"))
+    lpn = torch.cat([torch.zeros(phase, device="cuda"), lpn])[phase:]
+    m = (torch.rand(T + phase, device="cuda") < 0.7).to(torch.uint8)[phase:]
     R = torch.rand(J, device="cuda")
-    adv, grad, st = Guarded((J,), torch.float32), Guarded((T,), torch.float32), \
-        Guarded((4,), torch.float32)
+    adv, grad, st = Guarded((J,), torch.float32), \
+        Guarded((T,), torch.float32, offset=4 * phase), Guarded((4,), torch.float32)
     ws = Guarded((hdl.hdl_grpo_loss_workspace_bytes(),), torch.uint8)
     hdl.hdl_grpo_loss(lpn, lpo, m, toffs, R, goffs, advantages=adv.t, grad=grad.t, stats=st.t,
                       workspace=ws.t)

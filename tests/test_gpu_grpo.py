@@ -89,9 +89,13 @@ def test_grpo_paper_group(hdl):
 
 
 @pytest.mark.parametrize("shift", [1, 2, 3])
-def test_grpo_unaligned(hdl, shift):
+@pytest.mark.parametrize("grad_off", [None, 1, 2])
+def test_grpo_unaligned(hdl, shift, grad_off):
     """First trajectory starting at a token that is not a multiple of 4, and
-    buffers that are not 16-byte aligned: the scalar loading paths."""
+    buffers that are not 16-byte aligned: all four token streams one element
+    off (the phase-shifted vector path: grad_off 1), the gradient at another
+    offset (grad_off None: a fresh aligned buffer, or 2), which takes the
+    scalar path."""
     lpn, lpo, mask, toffs, R, goffs = make_batch(10 + shift, 30, 200)
     T = len(lpn)
     # `shift` leading tokens outside every trajectory, carrying no loss
@@ -99,10 +103,13 @@ def test_grpo_unaligned(hdl, shift):
     lpn2, lpo2, mask2 = pad(lpn, -1.0), pad(lpo, -1.0), pad(mask, 0)
     toffs2 = toffs + shift
     buf = lambda x: torch.from_numpy(np.concatenate([x[:1], x])).cuda()[1:]   # misalign
+    grad = None
+    if grad_off is not None:
+        grad = torch.full((len(lpn2) + grad_off,), 5.0, device="cuda")[grad_off:]
     adv, grad, stats = hdl.hdl_grpo_loss(buf(lpn2), buf(lpo2), buf(mask2),
                                          torch.from_numpy(toffs2).cuda(),
                                          torch.from_numpy(R).cuda(),
-                                         torch.from_numpy(goffs).cuda())
+                                         torch.from_numpy(goffs).cuda(), grad=grad)
     loss, g_ref, (n, cf, mr) = oracle.grpo_token_loss(
         lpn, lpo, mask, toffs, adv.cpu().numpy().astype(np.float64), decide_in=np.float32)
     st = stats.cpu().numpy()

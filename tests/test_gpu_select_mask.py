@@ -35,6 +35,19 @@ def make_roots(lengths, seed, tie_levels=None, nan_frac=0.0, invalid_frac=0.2):
     return delta, valid, offs
 
 
+def shifted(x: np.ndarray, off: int) -> torch.Tensor:
+    """x on the GPU starting `off` elements into a fresh (aligned) buffer."""
+    buf = torch.zeros(len(x) + off, dtype=torch.from_numpy(x[:0]).dtype, device="cuda")
+    buf[off:] = torch.from_numpy(x).cuda()
+    return buf[off:]
+
+
+# element offsets of (scores, validity): the same residue mod 4 keeps the
+# 16-byte path (shifted to the common phase), different ones take the
+# element-by-element path
+OFFSETS = [(1, 1), (3, 3), (1, 2), (2, 0)]
+
+
 def gpu_select(hdl, delta, valid, offs, k, **kw):
     d = torch.from_numpy(delta).cuda()
     v = None if valid is None else torch.from_numpy(valid).cuda()
@@ -124,23 +137,20 @@ def test_select_spacing_many_roots(hdl, gap_mode):
                                 lo=lo, hi=hi)
 
 
+@pytest.mark.parametrize("d_off,v_off", [(1, 1), (1, 2)])
 @pytest.mark.parametrize("n_roots", [7, 500])
 @pytest.mark.parametrize("gap_mode", [0, 1])
-def test_select_spacing_unaligned(hdl, n_roots, gap_mode):
-    """Scores / validity off their 16- / 4-byte alignment: the scalar paths
-    of both spacing modes, with few and with many roots."""
+def test_select_spacing_unaligned(hdl, n_roots, gap_mode, d_off, v_off):
+    """Scores / validity off their 16- / 4-byte alignment: both spacing modes
+    on the phase-shifted vector path and on the scalar path, with few and
+    with many roots."""
     lengths = list(np.random.default_rng(n_roots).integers(0, 2500, size=n_roots))
     delta, valid, offs = make_roots(lengths, 13, tie_levels=6)
     delta = add_spikes(delta, offs, 3)
-    N = len(delta)
-    d = torch.zeros(N + 1, dtype=torch.float32, device="cuda")
-    v = torch.zeros(N + 1, dtype=torch.uint8, device="cuda")
-    d[1:] = torch.from_numpy(delta).cuda()
-    v[1:] = torch.from_numpy(valid).cuda()
+    d, v = shifted(delta, d_off), shifted(valid, v_off)
     o = torch.from_numpy(offs).cuda()
     for min_gap in (2, 33):
-        bp, ns, bd = hdl.hdl_select_branches(d[1:], v[1:], o, 16, min_gap=min_gap,
-                                             gap_mode=gap_mode)
+        bp, ns, bd = hdl.hdl_select_branches(d, v, o, 16, min_gap=min_gap, gap_mode=gap_mode)
         pos, nsel, val = oracle.select_branches(delta.astype(np.float64), valid, offs, 16,
                                                 min_gap=min_gap, gap_mode=gap_mode)
         assert np.array_equal(ns.cpu().numpy(), nsel)
@@ -230,41 +240,38 @@ def test_suffix_mask(hdl, seed, n_cont, max_len):
 
 
 def test_suffix_mask_unaligned_and_offset_range(hdl):
-    """Byte path (mask not 16-byte aligned) and a range that starts and ends
-    mid-buffer: bytes outside the continuations stay untouched."""
+    """Mask and validity bytes at the same offset from 16-byte alignment (the
+    phase-shifted vector path), at different ones (the byte path), and a
+    range that starts and ends mid-buffer: bytes outside the continuations
+    stay untouched."""
     br, offs, valid = mask_case(3, 40, 200)
     total = int(offs[-1])
     shift = 5
-    offs2 = offs + shift
-    buf = torch.full((total + 2 * shift + 1,), 7, dtype=torch.uint8, device="cuda")
-    vbuf = torch.zeros_like(buf)
-    vbuf[shift:shift + total] = torch.from_numpy(valid).cuda()
+    L = total + 2 * shift
     ref = oracle.suffix_mask(br, offs, valid)
-    for base in (0, 1):            # base 1: neither buffer is 16-byte aligned
-        mview = buf[base:]
-        vview = vbuf[base:]
-        buf.fill_(7)
-        o = torch.from_numpy(offs2 - base).cuda()
-        hdl.hdl_suffix_mask(torch.from_numpy(br).cuda(), o, vview, mask=mview)
-        got = buf.cpu().numpy()
-        lo = shift
-        assert np.all(got[:lo] == 7) and np.all(got[lo + total:] == 7)
-        assert np.array_equal(got[lo:lo + total], ref)
+    o = torch.from_numpy(offs + shift).cuda()
+    for mbase, vbase in ((0, 0), (1, 1), (7, 7), (1, 3), (0, 9)):
+        mbuf = torch.full((L + mbase,), 7, dtype=torch.uint8, device="cuda")
+        vbuf = torch.zeros(L + vbase, dtype=torch.uint8, device="cuda")
+        vbuf[vbase + shift:vbase + shift + total] = torch.from_numpy(valid).cuda()
+        hdl.hdl_suffix_mask(torch.from_numpy(br).cuda(), o, vbuf[vbase:], mask=mbuf[mbase:])
+        got = mbuf[mbase:].cpu().numpy()
+        assert np.all(got[:shift] == 7) and np.all(got[shift + total:] == 7)
+        assert np.array_equal(got[shift:shift + total], ref)
 
 
+@pytest.mark.parametrize("d_off,v_off", OFFSETS)
 @pytest.mark.parametrize("n_roots", [5, 600])
-def test_select_unaligned_buffers(hdl, n_roots):
-    """Scores / validity not 16- / 4-byte aligned: the scalar loading path."""
+def test_select_unaligned_buffers(hdl, n_roots, d_off, v_off):
+    """Scores / validity off their 16- / 4-byte alignment: the phase-shifted
+    vector path when both are off by the same amount, else the scalar path."""
     lengths = list(np.random.default_rng(n_roots).integers(0, 500, size=n_roots))
     delta, valid, offs = make_roots(lengths, 12, tie_levels=5)
-    N = len(delta)
-    d = torch.zeros(N + 1, dtype=torch.float32, device="cuda")
-    v = torch.zeros(N + 1, dtype=torch.uint8, device="cuda")
-    d[1:] = torch.from_numpy(delta).cuda()
-    v[1:] = torch.from_numpy(valid).cuda()
-    bp, ns, bd = hdl.hdl_select_branches(d[1:], v[1:], torch.from_numpy(offs).cuda(), 8)
+    bp, ns, bd = hdl.hdl_select_branches(shifted(delta, d_off), shifted(valid, v_off),
+                                         torch.from_numpy(offs).cuda(), 8)
     pos, nsel, val = oracle.select_branches(delta.astype(np.float64), valid, offs, 8)
     assert np.array_equal(ns.cpu().numpy(), nsel) and np.array_equal(bp.cpu().numpy(), pos)
+    assert np.array_equal(bd.cpu().numpy().astype(np.float64), val, equal_nan=True)
 
 
 _SPLIT_SCRIPT = r"""
