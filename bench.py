@@ -41,7 +41,8 @@ def parse():
     p.add_argument("--steps", type=int, default=10)
     p.add_argument("--warmup", type=int, default=3)
     p.add_argument("--workload", default="code",
-                   help="tiny | math | code | agent | sweep_V<vocab>_N<tokens>")
+                   help="tiny | math | code | agent | sweep_V<vocab>_N<tokens>; a _f32 suffix "
+                        "(math_f32) gives fp32 hidden states and LM head (tf32 products)")
     p.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--graph", action="store_true",
@@ -66,6 +67,8 @@ def spec_for(name: str, seed: int) -> hdl_synth.Spec:
     import dataclasses
     if name in hdl_synth.SPECS:
         return dataclasses.replace(hdl_synth.SPECS[name], seed=seed)
+    if name.endswith("_f32") and name[:-4] in hdl_synth.SPECS:   # fp32 states: tf32 products
+        return dataclasses.replace(hdl_synth.SPECS[name[:-4]], name=name, dtype="f32", seed=seed)
     if name.startswith("sweep_V"):
         v, n = name[len("sweep_V"):].split("_N")
         return hdl_synth.sweep_spec(int(v), int(n), seed=seed)

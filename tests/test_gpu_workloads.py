@@ -1,10 +1,13 @@
 """The five workloads (tiny, math, code, agent, roofline sweep) at their full
-sizes, in the launch configuration the bench times.
+sizes, in the launch configuration the bench times, and the math workload
+with fp32 states (the tf32 path at a large shape).
 
 tiny and math: the oracle scores every token, so log-probs, scores and the
 end-to-end branch sets are compared in full.  code, agent and the sweep: the
 oracle scores sampled tokens one by one (first, last, random), and selection,
 allocation and masks are compared bit-exactly on the device's own scores."""
+import dataclasses
+
 import numpy as np
 import pytest
 import torch
@@ -77,15 +80,22 @@ def test_workload_full_oracle(hdl, name):
     check_downstream_exact(wl, out)
 
 
-SAMPLED = ["code", "agent", ("sweep", 32000, 8192), ("sweep", 256000, 262144),
+SAMPLED = ["code", "agent", "math_f32", ("sweep", 32000, 8192), ("sweep", 256000, 262144),
            ("sweep", 128256, 131072)]
+
+
+def sampled_spec(which):
+    if isinstance(which, tuple):
+        return hdl_synth.sweep_spec(which[1], which[2])
+    if which.endswith("_f32"):   # fp32 hidden states and LM head: tf32 products
+        return dataclasses.replace(hdl_synth.SPECS[which[:-4]], name=which, dtype="f32")
+    return hdl_synth.SPECS[which]
 
 
 @pytest.mark.parametrize("which", SAMPLED, ids=lambda w: w if isinstance(w, str) else
                          f"sweep_V{w[1]}_N{w[2]}")
 def test_workload_sampled(hdl, which):
-    spec = (hdl_synth.SPECS[which] if isinstance(which, str)
-            else hdl_synth.sweep_spec(which[1], which[2]))
+    spec = sampled_spec(which)
     wl = hdl_synth.generate(spec, device="cuda")
     out = run_path(hdl, wl)
     rows = sample_rows(wl.n_tokens, 40, seed=spec.d)
