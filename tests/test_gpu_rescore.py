@@ -60,6 +60,23 @@ def test_rescore_shapes(hdl, n, d, V, dt):
         assert np.all(r0 == 0.0)
 
 
+@pytest.mark.parametrize("V", [257, 1000, 4097, 32000])
+def test_rescore_targets_at_the_vocabulary_edges(hdl, V):
+    """Targets in the first column, the last column (inside the masked tail
+    of a partial 256-column tile), the last column of a full tile and the
+    first of the next, and the first and last columns of a vocabulary chunk:
+    every gather position the epilogue special-cases."""
+    spec = hdl_synth.small_spec(f"edge{V}", n_roots=1, t_lo=260, t_hi=260, d=128, vocab=V,
+                                seed=V)
+    wl = hdl_synth.generate(spec, device="cuda")
+    cols = [0, V - 1, min(255, V - 1), min(256, V - 1), min(4095, V - 1), min(4096, V - 1),
+            V // 2]
+    y = torch.tensor([cols[i % len(cols)] for i in range(wl.n_tokens)], dtype=torch.int32,
+                     device="cuda")
+    wl.targets.copy_(y)
+    run_and_check(hdl, wl, f"edges V={V}")
+
+
 def test_rescore_identical_contexts_bitwise(hdl):
     """Delta = 0 exactly when both contexts carry the same hidden states, and
     the two log-prob rows are bit-identical (same arithmetic for both)."""
