@@ -80,8 +80,10 @@ def test_workload_full_oracle(hdl, name):
     check_downstream_exact(wl, out)
 
 
+# the last entry is four times the largest workload: 2^20 tokens per context,
+# 4.3 G elements (8.6 GB) per context, past every 32-bit element count
 SAMPLED = ["code", "agent", "math_f32", ("sweep", 32000, 8192), ("sweep", 256000, 262144),
-           ("sweep", 128256, 131072)]
+           ("sweep", 128256, 131072), ("sweep", 32000, 1 << 20)]
 
 
 def sampled_spec(which):
