@@ -251,10 +251,12 @@ def aggregate_value(world: int, n_tokens_per_rank: int, steps: int, max_ms: floa
     return world * n_tokens_per_rank * steps / (max_ms / 1e3)
 
 
-def cpu_oracle_sample(wl, seconds: float, rng_seed: int = 0):
+def cpu_oracle_sample(wl, seconds: float, rng_seed: int = 0, gpu_logp=None):
     """Time the fp64 oracle on sampled tokens of the workload: log-probs of
     both contexts for a growing sample until ``seconds`` of CPU work, plus
-    selection / allocation / masks over the whole workload (on its scores)."""
+    selection / allocation / masks over the whole workload (on its scores).
+    With ``gpu_logp`` (the bench's own log-probs of both contexts, host
+    arrays), the sampled tokens' oracle values also give a parity figure."""
     import oracle
 
     def to_f64(t):  # exact widening of the bf16 / fp32 inputs
@@ -268,6 +270,7 @@ def cpu_oracle_sample(wl, seconds: float, rng_seed: int = 0):
     rng = np.random.default_rng(rng_seed)
     done, t_lp, block = 0, 0.0, 8
     delta_s = []
+    worst, within = 0.0, True
     while t_lp < seconds and done < N:
         rows = np.sort(rng.choice(N, size=min(block, N - done), replace=False))
         idx = torch.from_numpy(rows).to(wl.h_orig.device)
@@ -278,6 +281,11 @@ def cpu_oracle_sample(wl, seconds: float, rng_seed: int = 0):
         lp1 = oracle.target_logprobs(h1, W, y_all[rows])
         delta_s.append(oracle.hindsight_divergence(lp1, lp0))
         t_lp += time.perf_counter() - t0
+        if gpu_logp is not None:
+            for got, ref in ((gpu_logp[0][rows], lp0), (gpu_logp[1][rows], lp1)):
+                err = np.abs(got.astype(np.float64) - ref)
+                worst = max(worst, float(err.max()))
+                within = within and bool(np.all(err <= 1e-3 + 1e-3 * np.abs(ref)))
         done += len(rows)
         block = min(block * 2, 256)
     del W
@@ -291,12 +299,16 @@ def cpu_oracle_sample(wl, seconds: float, rng_seed: int = 0):
     oracle.suffix_mask(cb, wl.cont_offsets.cpu().numpy(), wl.cont_valid.cpu().numpy())
     t_down = time.perf_counter() - t0
     per_token = t_lp / done + t_down / N
-    return {"value": 1.0 / per_token, "unit": "root tokens/s",
-            "cores": int(os.environ.get("OPENBLAS_NUM_THREADS", os.cpu_count() or 1)),
-            "kind": "oracle",
-            "sample": (f"log-probs of both contexts for {done} random tokens of {N} "
-                       f"({t_lp:.1f} s), selection + allocation + masks over all {N} "
-                       f"tokens ({t_down:.2f} s); per-token times added")}
+    out = {"value": 1.0 / per_token, "unit": "root tokens/s",
+           "cores": int(os.environ.get("OPENBLAS_NUM_THREADS", os.cpu_count() or 1)),
+           "kind": "oracle",
+           "sample": (f"log-probs of both contexts for {done} random tokens of {N} "
+                      f"({t_lp:.1f} s), selection + allocation + masks over all {N} "
+                      f"tokens ({t_down:.2f} s); per-token times added")}
+    if gpu_logp is not None:
+        out["parity"] = {"tokens": done, "max_abs_err_logp": worst,
+                         "tolerance": "1e-3 + 1e-3 |ref|", "within": within}
+    return out
 
 
 def run_reference(args, world, rank):
@@ -476,7 +488,9 @@ def run_gpu(args, world, rank, local):
 
     cpu = None
     if rank == 0 and not args.no_cpu:
-        cpu = cpu_oracle_sample(wl, args.cpu_seconds)
+        # the timed steps' own log-probs, checked on the oracle's sampled tokens
+        cpu = cpu_oracle_sample(wl, args.cpu_seconds,
+                                gpu_logp=(path.lp0.cpu().numpy(), path.lp1.cpu().numpy()))
 
     if rank != 0:
         return

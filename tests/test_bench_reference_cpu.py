@@ -57,3 +57,27 @@ def test_reference_arm_two_ranks():
     lines = json_lines(r.stdout)
     assert len(lines) == 1
     check_line(lines[0], 2)
+
+
+def test_cpu_baseline_parity_figure():
+    """The CPU-baseline leg checks the bench's own log-probs on the tokens it
+    samples: values equal to the oracle's are within tolerance, and a planted
+    error of 0.05 in one context is reported."""
+    import numpy as np
+    import sys
+    sys.path.insert(0, ROOT)
+    import bench
+    import hdl_synth
+    import oracle
+    wl = hdl_synth.generate(hdl_synth.SPECS["tiny"], device="cpu")
+    W = oracle.widen(wl.w.numpy(), "f32")
+    y = wl.targets.numpy()
+    lp0 = oracle.target_logprobs(oracle.widen(wl.h_orig.numpy(), "f32"), W, y)
+    lp1 = oracle.target_logprobs(oracle.widen(wl.h_hind.numpy(), "f32"), W, y)
+    good = bench.cpu_oracle_sample(wl, 0.2, gpu_logp=(lp0, lp1))
+    assert good["parity"]["within"] and good["parity"]["max_abs_err_logp"] < 1e-9
+    assert good["parity"]["tokens"] > 0
+    bad = bench.cpu_oracle_sample(wl, 0.2, gpu_logp=(lp0, lp1 + 0.05))
+    assert not bad["parity"]["within"]
+    assert abs(bad["parity"]["max_abs_err_logp"] - 0.05) < 1e-9
+    assert "parity" not in bench.cpu_oracle_sample(wl, 0.1)

@@ -42,6 +42,7 @@ def test_gb300_arm_line():
     c = d["cpu_baseline"]
     assert c["kind"] == "oracle" and num(c["value"]) and c["value"] > 0
     assert isinstance(c["cores"], int) and c["cores"] >= 1 and c["sample"]
+    assert c["parity"]["within"] is True and c["parity"]["tokens"] > 0   # the timed outputs
     e = d["e2e"]
     assert num(e["value"]) and e["value"] > 0 and e["unit"] == d["unit"]
     assert e["h2d_bytes_per_step"] > 0 and e["d2h_bytes_per_step"] > 0
