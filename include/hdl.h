@@ -237,8 +237,11 @@ HDL_API hdl_status hdl_grpo_loss(const float* logp_new, const float* logp_old,
  *     (e.g. at d = 3584, vocab = 152064 about 28,000 tokens fit; at d = 2048,
  *     vocab = 32000 about 250,000).
  *   - The first call on a device looks up the array's device address (with
- *     that device current) and caches it; make that first call before any
- *     stream capture.
+ *     that device current) and caches it, keyed on the context's
+ *     process-unique id; make that first call before any stream capture.  A
+ *     call from a new context of the device (for instance after
+ *     cudaDeviceReset re-created the primary context) looks the address up
+ *     again, so that call, too, should come before any capture.
  *   - Every call on a device shares the one array and leaves its contents
  *     behind; each call clears the status word it needs.  Calls that overlap
  *     on the GPU (e.g. on two streams at once) race on the array: serialise

@@ -117,19 +117,6 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* m,
       : "memory");
 }
 
-// Multicast variant: the box lands at the same shared-memory offset in every
-// CTA of the cluster named in `mask`, and each of them gets the transaction
-// bytes on its mbarrier at offset `bar`.
-__device__ __forceinline__ void tma_load_2d_multicast(uint32_t dst, const CUtensorMap* m,
-                                                      int32_t c0, int32_t c1, uint32_t bar,
-                                                      uint16_t mask) {
-  asm volatile(
-      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
-      ".multicast::cluster [%0], [%1, {%2, %3}], [%4], %5;" ::"r"(dst),
-      "l"(reinterpret_cast<uint64_t>(m)), "r"(c0), "r"(c1), "r"(bar), "h"(mask)
-      : "memory");
-}
-
 // CTA-pair variant: the box lands in this CTA's shared memory and its
 // transaction bytes are signalled on `bar_cluster`, an mbarrier that may sit
 // in either CTA of the pair (a shared::cluster address, e.g. from mapa).
@@ -274,18 +261,21 @@ __device__ __forceinline__ void tc_mma_pair(uint32_t d_tmem, uint64_t adesc, uin
   }
 }
 
-// Pair-MMA completion: arrive on the mbarrier at offset `bar` of every CTA
-// in `mask` once the pair MMAs issued so far have completed.
-__device__ __forceinline__ void tc_commit_pair_multicast(uint32_t bar, uint16_t mask) {
-  asm volatile(
-      "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64"
-      " [%0], %1;" ::"r"(bar), "h"(mask)
-      : "memory");
-}
+// Pair-MMA completion: arrive once on the mbarrier at `bar` (a shared::cluster
+// address: this CTA's own, or the peer's from mapa) when the pair MMAs issued
+// so far by this thread have completed.
 __device__ __forceinline__ void tc_commit_pair(uint32_t bar) {
   asm volatile("tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
                    bar)
                : "memory");
+}
+// The same completion signalled to the mbarrier at offset `bar` in both CTAs
+// of the pair (issued by the even CTA): one commit per CTA.
+__device__ __forceinline__ void tc_commit_pair_both(uint32_t bar) {
+  tc_commit_pair(bar);
+  uint32_t peer;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, 1;" : "=r"(peer) : "r"(bar));
+  tc_commit_pair(peer);
 }
 
 // Arrive on `bar` once every tcgen05 operation issued so far by this thread
@@ -293,15 +283,6 @@ __device__ __forceinline__ void tc_commit_pair(uint32_t bar) {
 __device__ __forceinline__ void tc_commit(uint32_t bar) {
   asm volatile(
       "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
-      : "memory");
-}
-
-// As tc_commit, but arrives on the mbarrier at offset `bar` of every CTA of
-// the cluster named in `mask`.
-__device__ __forceinline__ void tc_commit_multicast(uint32_t bar, uint16_t mask) {
-  asm volatile(
-      "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64"
-      " [%0], %1;" ::"r"(bar), "h"(mask)
       : "memory");
 }
 

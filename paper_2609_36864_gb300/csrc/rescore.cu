@@ -16,8 +16,8 @@
 // the ~150 concurrently running units touch stay in L2 -- W is then streamed
 // from DRAM once per group instead of once per M-tile.
 //
-// Roles inside a CTA of 192 threads (shown for the single-CTA organisation;
-// Cfg below describes the CTA-pair ones, the default):
+// Roles inside a CTA of 192 threads (shown for the single-CTA organisation,
+// the default; Cfg below describes the CTA-pair one):
 //   warp 0      TMA producer: H tile (128 x 128 B) + W tile (256 x 128 B) per
 //               K step into a kStages-deep shared-memory ring;
 //   warp 1      TMEM allocator and MMA issuer (one thread): 4 x
@@ -56,7 +56,7 @@ constexpr int kPairsInFlight = 76;      // CTA pairs resident on 152 SMs
 #define HDL_GROUP_M 32
 #endif
 constexpr int kGroupM = HDL_GROUP_M; // M-tiles per rasterisation group (even)
-constexpr int kDefaultMode = 1;      // CTA organisation, see Cfg
+constexpr int kDefaultMode = 0;      // CTA organisation, see Cfg
 constexpr int kThreads = 192;
 static_assert(kGroupM % 2 == 0 && kGroupM >= 2, "group of M-tiles must be even");
 constexpr int kAStage = kBM * kRowBytes;        // 16 KiB
@@ -64,19 +64,18 @@ constexpr int kMmaPerStage = kRowBytes / 32;    // 32 bytes of K per MMA
 constexpr int kTmemCols = 2 * kBN;              // two accumulator buffers
 
 // CTA organisation of the kernel:
-//   mode 0  one CTA per unit, 128 x 256 MMA (cta_group::1), whole W tiles;
-//   mode 1  clusters of two CTAs on neighbouring M-tiles; each loads half of
-//           every W tile and multicasts it into both CTAs (1-CTA MMAs);
+//   mode 0  one CTA per unit, 128 x 256 MMA (cta_group::1), whole W tiles
+//           (the default);
 //   mode 2  clusters of two CTAs running the 256 x 256 pair MMA
 //           (cta_group::2): each CTA holds its 128 H rows and one 128-row
 //           half of the W tile, so a stage is 32 KiB and the ring 6 deep.
-// (Clusters of four were measured too: only 36 fit at once, leaving 8 SMs
-// idle, and they were not faster.)
+// Every copy is an ordinary tile load into the issuing CTA's own shared
+// memory; no load is shared between CTAs.
 template <int M>
 struct Cfg {
-  static constexpr bool kCluster = M != 0;
-  static constexpr int kCS = M != 0 ? 2 : 1;    // CTAs per cluster
-  static constexpr bool kMulticast = M == 1;     // W halves multicast
+  static_assert(M == 0 || M == 2, "CTA organisation 0 or 2");
+  static constexpr bool kCluster = M == 2;
+  static constexpr int kCS = M == 2 ? 2 : 1;    // CTAs per cluster
   static constexpr int kBRows = M == 2 ? kBN / 2 : kBN;  // W rows held per CTA
   static constexpr int kBStage = kBRows * kRowBytes;
   static constexpr int kStageBytes = kAStage + kBStage;
@@ -182,12 +181,11 @@ __device__ __forceinline__ void lse_fold_ent(const float (&x)[32], float& m2, fl
   m2 = m_new;
 }
 
-// One persistent kernel for both contexts.  See Cfg for the three CTA
-// organisations.  In the cluster modes a stage may be refilled only once the
-// MMAs of the pair are done with it (mode 1: both CTAs' commits arrive on the
-// stage's empty barrier in both CTAs; mode 2: the even CTA's pair-MMA commit
-// arrives in both), and in mode 2 both CTAs' copies are counted on the even
-// CTA's full barrier and both epilogues release TMEM to the even CTA.
+// One persistent kernel for both contexts.  See Cfg for the two CTA
+// organisations.  In the pair mode a stage may be refilled only once the pair
+// MMAs are done with it (the even CTA commits to the stage's empty barrier in
+// each CTA), both CTAs' copies are counted on the even CTA's full barrier and
+// both epilogues release TMEM to the even CTA.
 template <bool kTf32, int M, bool kEnt>
 __global__ void __launch_bounds__(kThreads, 1)
     rescore_lse_kernel(const __grid_constant__ CUtensorMap tm_h0,
@@ -221,7 +219,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (threadIdx.x == 0) {
     for (int s = 0; s < C::kStages; ++s) {
       mbar_init(full_bar(s), 1);
-      mbar_init(empty_bar(s), C::kMulticast ? C::kCS : 1);
+      mbar_init(empty_bar(s), 1);
     }
     for (int b = 0; b < 2; ++b) {
       mbar_init(tfull_bar(b), 1);
@@ -274,13 +272,6 @@ __global__ void __launch_bounds__(kThreads, 1)
               if (leader) mbar_arrive_expect_tx(full_bar(stage), 2 * C::kStageBytes);
               tma_load_2d_pair(dA, tmA, kx, w.row0, fb);
               tma_load_2d_pair(dB, &tm_w, kx, vt * kBN + rank * (kBN / 2), fb);
-            } else if constexpr (C::kMulticast) {
-              constexpr int part = kBN / C::kCS;   // W rows this CTA fetches
-              mbar_arrive_expect_tx(full_bar(stage), C::kStageBytes);
-              tma_load_2d(dA, tmA, kx, w.row0, full_bar(stage));
-              tma_load_2d_multicast(dB + static_cast<uint32_t>(rank * part * kRowBytes), &tm_w,
-                                    kx, vt * kBN + rank * part, full_bar(stage),
-                                    static_cast<uint16_t>((1u << C::kCS) - 1u));
             } else {
               mbar_arrive_expect_tx(full_bar(stage), C::kStageBytes);
               tma_load_2d(dA, tmA, kx, w.row0, full_bar(stage));
@@ -347,9 +338,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 tc_mma<kTf32>(d_tmem, ad, bd, idesc, acc);
             }
             if constexpr (M == 2)
-              tc_commit_pair_multicast(empty_bar(stage), 0x3);
-            else if constexpr (C::kMulticast)
-              tc_commit_multicast(empty_bar(stage), static_cast<uint16_t>((1u << C::kCS) - 1u));
+              tc_commit_pair_both(empty_bar(stage));
             else
               tc_commit(empty_bar(stage));
             if (++stage == C::kStages) {
@@ -359,7 +348,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
           if (ok) {
             if constexpr (M == 2)
-              tc_commit_pair_multicast(tfull_bar(buf), 0x3);
+              tc_commit_pair_both(tfull_bar(buf));
             else
               tc_commit(tfull_bar(buf));
           }
@@ -731,13 +720,13 @@ hdl_status launch_rescore(const CUtensorMap& tm_h0, const CUtensorMap& tm_h1,
   return HDL_OK;
 }
 
-// CTA organisation (see Cfg): kDefaultMode unless HDL_RESCORE_MODE = 0, 1 or
-// 2 is set in the environment (a tuning override; every mode gives the same
+// CTA organisation (see Cfg): kDefaultMode unless HDL_RESCORE_MODE = 0 or 2
+// is set in the environment (a tuning override; both modes give the same
 // results bit for bit).
 int rescore_mode() {
   static const int mode = [] {
     const char* e = std::getenv("HDL_RESCORE_MODE");
-    if (e && (e[0] == '0' || e[0] == '1' || e[0] == '2') && e[1] == '\0') return e[0] - '0';
+    if (e && (e[0] == '0' || e[0] == '2') && e[1] == '\0') return e[0] - '0';
     return kDefaultMode;
   }();
   return mode;
@@ -839,15 +828,12 @@ extern "C" hdl_status hdl_rescore_ex(const void* h_orig, const void* h_hind,
   if (ent)
     ls = tf32 ? launch_rescore<true, kDefaultMode, true>(tm_h0, tm_h1, tm_w, a, sms, st)
               : launch_rescore<false, kDefaultMode, true>(tm_h0, tm_h1, tm_w, a, sms, st);
-  else if (mode == 0)
-    ls = tf32 ? launch_rescore<true, 0, false>(tm_h0, tm_h1, tm_w, a, sms, st)
-              : launch_rescore<false, 0, false>(tm_h0, tm_h1, tm_w, a, sms, st);
   else if (mode == 2)
     ls = tf32 ? launch_rescore<true, 2, false>(tm_h0, tm_h1, tm_w, a, sms, st)
               : launch_rescore<false, 2, false>(tm_h0, tm_h1, tm_w, a, sms, st);
   else
-    ls = tf32 ? launch_rescore<true, 1, false>(tm_h0, tm_h1, tm_w, a, sms, st)
-              : launch_rescore<false, 1, false>(tm_h0, tm_h1, tm_w, a, sms, st);
+    ls = tf32 ? launch_rescore<true, 0, false>(tm_h0, tm_h1, tm_w, a, sms, st)
+              : launch_rescore<false, 0, false>(tm_h0, tm_h1, tm_w, a, sms, st);
   if (ls != HDL_OK) return ls;
   if (launch_status() != HDL_OK) return HDL_ERR_CUDA;
 
@@ -885,26 +871,58 @@ extern "C" hdl_status hdl_device_status(const void* workspace, size_t workspace_
 // ---------------------------------------------------------------------------
 // Allocation-free variant: the scratch lives in one file-scope device array.
 // Host code may not use the array's name as a device address (it is a
-// host-side stand-in); its device address is looked up once per device.
+// host-side stand-in); its device address is looked up once per device and
+// context, with that device current.
 static __device__ __align__(256) uint8_t g_static_scratch[HDL_STATIC_SCRATCH_BYTES];
 
 namespace {
 constexpr int kMaxDevices = 128;
 std::mutex g_scratch_mu;
-void* g_scratch_addr[kMaxDevices] = {};
+struct ScratchSlot {
+  unsigned long long ctx_id;   // the context the address belongs to (0 = none yet)
+  void* addr;
+};
+ScratchSlot g_scratch[kMaxDevices] = {};
 
+// Process-unique id of the calling thread's current context (never reused,
+// unlike a context handle, so a context re-created after cudaDeviceReset has
+// a new one); 0 if it cannot be read.
+unsigned long long current_context_id() {
+  static PFN_cuCtxGetId_v12000 get_id = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetId", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      get_id = reinterpret_cast<PFN_cuCtxGetId_v12000>(p);
+  });
+  unsigned long long id = 0;
+  if (!get_id || get_id(nullptr, &id) != CUDA_SUCCESS) return 0;
+  return id;
+}
+
+// The array's device address in the current device's current context.  The
+// address is cached per device together with the context's id; a call from
+// another context of the device (e.g. after cudaDeviceReset re-created the
+// primary context) looks it up again.
 hdl_status static_scratch_address(void** out) {
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess) return HDL_ERR_CUDA;
   if (dev < 0 || dev >= kMaxDevices) return HDL_ERR_UNSUPPORTED;
+  if (!ensure_context()) return HDL_ERR_CUDA;
+  const unsigned long long ctx = current_context_id();
   std::lock_guard<std::mutex> lock(g_scratch_mu);
-  if (g_scratch_addr[dev] == nullptr) {
+  ScratchSlot& slot = g_scratch[dev];
+  if (ctx == 0 || slot.addr == nullptr || slot.ctx_id != ctx) {
     void* p = nullptr;
     if (cudaGetSymbolAddress(&p, g_static_scratch) != cudaSuccess || p == nullptr)
       return HDL_ERR_CUDA;
-    g_scratch_addr[dev] = p;
+    slot.addr = p;
+    slot.ctx_id = ctx;
   }
-  *out = g_scratch_addr[dev];
+  *out = slot.addr;
   return HDL_OK;
 }
 }  // namespace
