@@ -49,6 +49,10 @@ def parse():
                    help="capture one step in a CUDA graph and time its replays "
                         "(for launch-bound workloads such as tiny)")
     p.add_argument("--no-cpu", action="store_true")
+    p.add_argument("--no-extra", action="store_true",
+                   help="skip the kernel-only timings of the other large workloads that the "
+                        "default (code) run adds under 'workloads'")
+    p.add_argument("--extra-steps", type=int, default=5)
     p.add_argument("--cpu-seconds", type=float, default=12.0)
     p.add_argument("--digest", nargs="+", default=None, metavar="FILE",
                    help="print the comment-insensitive digest of csrc/FILE... and exit")
@@ -111,6 +115,25 @@ def committed_traffic(workload: str):
         if len(f) >= 4 and f[0] == workload and f[1] == digest:
             return float(f[2]) + float(f[3])
     return None
+
+
+def input_bytes(wl) -> int:
+    """Bytes of the step's large resident inputs: both contexts' states and W."""
+    return sum(t.numel() * t.element_size() for t in (wl.h_orig, wl.h_hind, wl.w))
+
+
+def workload_config(spec, wl, graph: bool) -> dict:
+    """The ``config`` of the JSON line, identical for both arms: the workload,
+    its sizes and how L2 is handled between timed steps."""
+    in_bytes = input_bytes(wl)
+    l2 = (f"inputs larger than L2 ({in_bytes / 2**30:.2f} GiB resident), steps back to back"
+          if in_bytes > 2 * L2_BYTES else
+          f"L2 flushed before every step (inputs {in_bytes / 2**20:.1f} MiB < 2 x L2); "
+          "only the steps are timed")
+    return {"workload": spec.name, "n_tokens": wl.n_tokens, "d": spec.d, "vocab": spec.vocab,
+            "launch": "CUDA graph replay of one step" if graph else "eager",
+            "roots": spec.n_roots, "k": spec.k, "conts": int(wl.cont_offsets.numel() - 1),
+            "context_rows_per_step": 2 * wl.n_tokens, "l2": l2}
 
 
 class ClockSampler:
@@ -299,7 +322,7 @@ def cpu_oracle_sample(wl, seconds: float, rng_seed: int = 0, gpu_logp=None):
     oracle.suffix_mask(cb, wl.cont_offsets.cpu().numpy(), wl.cont_valid.cpu().numpy())
     t_down = time.perf_counter() - t0
     per_token = t_lp / done + t_down / N
-    out = {"value": 1.0 / per_token, "unit": "root tokens/s",
+    out = {"value": 1.0 / per_token, "unit": "root tokens/s", "sample_fraction": done / N,
            "cores": int(os.environ.get("OPENBLAS_NUM_THREADS", os.cpu_count() or 1)),
            "kind": "oracle",
            "sample": (f"log-probs of both contexts for {done} random tokens of {N} "
@@ -308,6 +331,85 @@ def cpu_oracle_sample(wl, seconds: float, rng_seed: int = 0, gpu_logp=None):
     if gpu_logp is not None:
         out["parity"] = {"tokens": done, "max_abs_err_logp": worst,
                          "tolerance": "1e-3 + 1e-3 |ref|", "within": within}
+    return out
+
+
+def cpu_oracle_parity(wl, lp0, lp1, count: int = 40, seed: int = 0):
+    """Oracle log-probs of both contexts on ``count`` sampled tokens (first,
+    last, random) against the GPU's (host arrays): tokens, largest error and
+    whether all are within 1e-3 + 1e-3 |ref|."""
+    import oracle
+
+    def to_f64(t):
+        t = t.detach().cpu().contiguous()
+        if t.dtype == torch.bfloat16:
+            return oracle.widen(t.view(torch.int16).numpy(), "bf16")
+        return oracle.widen(t.numpy(), "f32")
+    N = wl.n_tokens
+    rng = np.random.default_rng(seed)
+    rows = np.array(sorted({0, N - 1} | set(rng.integers(0, N, size=count - 2).tolist())))
+    idx = torch.from_numpy(rows).to(wl.h_orig.device)
+    W = to_f64(wl.w)
+    y = wl.targets.cpu().numpy()[rows]
+    worst, within = 0.0, True
+    for got, h in ((lp0, wl.h_orig), (lp1, wl.h_hind)):
+        ref = oracle.target_logprobs(to_f64(h.index_select(0, idx)), W, y)
+        err = np.abs(got[rows].astype(np.float64) - ref)
+        worst = max(worst, float(err.max()))
+        within = within and bool(np.all(err <= 1e-3 + 1e-3 * np.abs(ref)))
+    return {"tokens": int(len(rows)), "max_abs_err_logp": worst,
+            "tolerance": "1e-3 + 1e-3 |ref|", "within": within}
+
+
+# The other workloads the tensor-peak target is stated on, timed after the
+# default one (kernel only: the fused re-scoring call, inputs resident).
+EXTRA_WORKLOADS = ("agent", "sweep_V32000_N262144", "sweep_V256000_N262144")
+
+
+def time_extra_workloads(hdl, args, local, check: bool):
+    burst, sustained, _, src = peaks()
+    dev = torch.device("cuda", local)
+    stream = torch.cuda.current_stream()
+    out = []
+    for name in EXTRA_WORKLOADS:
+        spec = spec_for(name, seed=0)
+        wl = hdl_synth.generate(spec, device=dev)
+        N, d, V = wl.n_tokens, spec.d, spec.vocab
+        lp0 = torch.empty(N, dtype=torch.float32, device=dev)
+        lp1, delta = torch.empty_like(lp0), torch.empty_like(lp0)
+        ws = torch.empty(hdl.hdl_rescore_workspace_bytes(N, d, V, wl.h_orig.dtype),
+                         dtype=torch.uint8, device=dev)
+        call = lambda: hdl.hdl_rescore(wl.h_orig, wl.h_hind, wl.w, wl.targets, lp0, lp1,
+                                       delta, ws, stream=stream)
+        for _ in range(2):
+            call()
+        torch.cuda.synchronize()
+        steps = args.extra_steps
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+              for _ in range(steps)]
+        clocks = ClockSampler(local)
+        clocks.start()
+        for a, b_ in ev:            # inputs are larger than L2: back to back
+            a.record(stream)
+            call()
+            b_.record(stream)
+        torch.cuda.synchronize()
+        clk = clocks.stop()
+        code, raw = hdl.hdl_device_status(ws, stream)
+        assert code == hdl.HDL_OK, (name, code, raw)
+        ms = float(np.mean([a.elapsed_time(b_) for a, b_ in ev]))
+        tflops = 2.0 * (2 * N) * d * V / (ms / 1e3) / 1e12
+        rec = {"workload": name, "n_tokens": N, "d": d, "vocab": V, "steps": steps,
+               "rescore_ms": ms, "root_tokens_per_s": N / (ms / 1e3), "tflops": tflops,
+               "frac_sustained": tflops / sustained, "frac_burst": tflops / burst,
+               "peak_kind": f"bf16 ({src})", "clocks": clk,
+               "tflops_per_ghz": (tflops / (clk["sm_mhz"] / 1e3)
+                                  if clk.get("sm_mhz") else None)}
+        if check:
+            rec["cpu_check"] = cpu_oracle_parity(wl, lp0.cpu().numpy(), lp1.cpu().numpy())
+        out.append(rec)
+        del wl, lp0, lp1, delta, ws, call
+        torch.cuda.empty_cache()
     return out
 
 
@@ -332,8 +434,7 @@ def run_reference(args, world, rank):
             "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": 1e3 * wall / max(1, args.steps), "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-            "config": {"workload": spec.name, "n_tokens": wl.n_tokens, "d": spec.d,
-                       "vocab": spec.vocab, "roots": spec.n_roots, "k": spec.k},
+            "config": workload_config(spec, wl, args.graph),
             "cpu_baseline": cb,
             "e2e": {"value": value, "unit": "root tokens/s", "h2d_bytes_per_step": 0,
                     "d2h_bytes_per_step": 0}}
@@ -354,7 +455,7 @@ def run_gpu(args, world, rank, local):
     stream = torch.cuda.current_stream()
     N, d, V = wl.n_tokens, spec.d, spec.vocab
     flops = 2.0 * (2 * N) * d * V
-    in_bytes = sum(t.numel() * t.element_size() for t in (wl.h_orig, wl.h_hind, wl.w))
+    in_bytes = input_bytes(wl)
 
     for _ in range(max(args.warmup, 3)):
         path.rescore(stream)
@@ -419,10 +520,6 @@ def run_gpu(args, world, rank, local):
         first = {"sm_mhz": clk.get("sm_mhz"), "reasons": clk.get("reasons")}
         total_ms, rescore_ms, clk = timed_region()
         clk["remeasured_after"] = first
-    l2_note = (f"inputs larger than L2 ({in_bytes / 2**30:.2f} GiB resident), steps back to back"
-               if flush is None else
-               f"L2 flushed before every step (inputs {in_bytes / 2**20:.1f} MiB < 2 x L2); "
-               "only the steps are timed")
     value = aggregate_value(world, N, args.steps, total_ms)
 
     # ---- end to end: every step's inputs are copied host -> device from
@@ -492,6 +589,14 @@ def run_gpu(args, world, rank, local):
         cpu = cpu_oracle_sample(wl, args.cpu_seconds,
                                 gpu_logp=(path.lp0.cpu().numpy(), path.lp1.cpu().numpy()))
 
+    config = workload_config(spec, wl, args.graph)
+    extra = None
+    if world == 1 and spec.name == "code" and not args.no_extra:
+        # free the default workload, then the other large ones, one at a time
+        del path, wl, flush, graph
+        torch.cuda.empty_cache()
+        extra = time_extra_workloads(hdl, args, local, check=not args.no_cpu)
+
     if rank != 0:
         return
     burst, sustained, hbm, src = peaks()
@@ -513,11 +618,7 @@ def run_gpu(args, world, rank, local):
         "ms_per_step": total_ms / args.steps, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "bf16" if spec.dtype == "bf16" else "tf32",
         "data": "synthetic",
-        "config": {"workload": spec.name, "n_tokens": N, "d": d, "vocab": V,
-                   "launch": "CUDA graph replay of one step" if args.graph else "eager",
-                   "roots": spec.n_roots, "k": spec.k, "conts": path.C,
-                   "context_rows_per_step": 2 * N,
-                   "l2": l2_note},
+        "config": config,
         "tflops": flops * args.steps / (total_ms / 1e3) / 1e12,
         "pct_bf16_peak": 100.0 * (flops * args.steps / (total_ms / 1e3) / 1e12) / burst,
         "roofline": {"bound": "tensor", "kernel": "rescore_lse_kernel (+ merge)",
@@ -529,6 +630,8 @@ def run_gpu(args, world, rank, local):
         "cpu_baseline": cpu, "e2e": e2e, "clocks": clk,
         "gpu_launches": Path.LAUNCHES_PER_STEP * args.steps,
     }
+    if extra is not None:
+        line["workloads"] = extra
     print(json.dumps(line), flush=True)
 
 

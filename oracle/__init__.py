@@ -252,7 +252,7 @@ def group_advantages(rewards, group_offsets) -> np.ndarray:
 
 
 def grpo_token_loss(logp_new, logp_old, mask, traj_offsets, advantages,
-                    eps_low: float = 0.2, eps_high: float = 0.28, decide_in=np.float64):
+                    eps_low: float = 0.2, eps_high: float = 0.28):
     """Clipped policy loss aggregated over tokens (Section 4.1).
 
     For token t of trajectory j with mask m_t (Section 3.3's suffix-only mask):
@@ -260,12 +260,10 @@ def grpo_token_loss(logp_new, logp_old, mask, traj_offsets, advantages,
       obj_t = min(r_t A_j, clip(r_t, 1 - eps_low, 1 + eps_high) A_j)
       loss  = - sum_t m_t obj_t / sum_t m_t
     and grad_t = d loss / d logp_new_t, which is -m_t r_t A_j / sum m when the
-    unclipped term is the minimum (ties included) and 0 otherwise.
+    unclipped term is the minimum (ties included) and 0 otherwise.  Every
+    quantity, the choice of the minimum included, is taken in float64.
     Returns (loss, grad, stats) with stats = (masked tokens, fraction of masked
     tokens whose clipped term is strictly the minimum, mean masked ratio).
-    ``decide_in`` is the precision in which "which term is the minimum" is
-    decided (the values themselves stay float64): a GPU comparison passes
-    np.float32, the precision the kernel decides in.
     """
     lpn = np.asarray(logp_new, dtype=np.float64)
     lpo = np.asarray(logp_old, dtype=np.float64)
@@ -277,15 +275,10 @@ def grpo_token_loss(logp_new, logp_old, mask, traj_offsets, advantages,
     r = np.exp(lpn - lpo)
     unclipped = r * A
     clipped = np.clip(r, 1.0 - eps_low, 1.0 + eps_high) * A
-    obj = np.minimum(unclipped, clipped)
     n = int(m.sum())
     if n == 0:
         return 0.0, np.zeros(len(lpn)), (0, 0.0, 0.0)
-    loss = -obj[m].sum() / n
-    r_d = np.exp(lpn.astype(decide_in) - lpo.astype(decide_in))
-    A_d = A.astype(decide_in)
-    lo_d, hi_d = decide_in(1.0) - decide_in(eps_low), decide_in(1.0) + decide_in(eps_high)
-    active = (r_d * A_d) <= (np.clip(r_d, lo_d, hi_d) * A_d)
+    active = unclipped <= clipped            # the unclipped term is the minimum
     obj = np.where(active, unclipped, clipped)
     loss = -obj[m].sum() / n
     grad = np.where(m & active, -r * A / n, 0.0)

@@ -66,3 +66,43 @@ def check_selection_band(gpu_pos, gpu_nsel, ref_delta, valid, offs, k, band=SELE
         kth = ref_delta[offs[r] + pos[r, n - 1]]
         for t in a ^ b:
             assert abs(ref_delta[offs[r] + t] - kth) <= band, (r, t, ref_delta[offs[r] + t], kth)
+
+
+# GRPO: tokens closer than this many float32 ulps to a clip bound may be
+# decided either way by a float32 kernel (the float32 difference of the
+# log-probs is rounded, and CUDA's expf may differ from the exact ratio by
+# up to 2 ulp), so the float64 oracle's decision is not binding there.
+GRPO_DECISION_ULPS = 4
+
+
+def grpo_decided(lpn, lpo, eps_low=0.2, eps_high=0.28):
+    """Tokens whose ratio exp(lpn - lpo), taken in float64, lies more than
+    GRPO_DECISION_ULPS float32 ulps from 1 - eps_low and 1 + eps_high: there
+    a float32 kernel and the float64 oracle must pick the same term."""
+    r = np.exp(np.asarray(lpn, np.float64) - np.asarray(lpo, np.float64))
+    ok = np.ones(len(r), dtype=bool)
+    for b in (1.0 - eps_low, 1.0 + eps_high):
+        ok &= np.abs(r - b) > GRPO_DECISION_ULPS * float(np.spacing(np.float32(b)))
+    return ok
+
+
+def check_grpo(adv, grad, stats, lpn, lpo, mask, toffs, rewards, goffs, grad_slice=None):
+    """The GRPO update's outputs (host arrays) against the oracle, which
+    takes only the inputs: advantages within 1e-6, loss 1e-5 relative,
+    gradient 1e-5 of its largest entry on the tokens both sides must decide
+    alike; the clip fraction may differ by the undecided masked tokens."""
+    A_ref = oracle.group_advantages(rewards, goffs)
+    assert np.allclose(adv, A_ref, rtol=0, atol=1e-6), np.abs(adv - A_ref).max()
+    loss, g_ref, (n, clip_frac, mean_r) = oracle.grpo_token_loss(lpn, lpo, mask, toffs, A_ref)
+    assert stats[1] == n
+    assert abs(stats[0] - loss) <= 1e-5 * max(1.0, abs(loss)), (stats[0], loss)
+    ok = grpo_decided(lpn, lpo)
+    m = np.asarray(mask) != 0
+    undecided = int((m & ~ok).sum())
+    assert abs(stats[2] - clip_frac) <= 1e-6 + undecided / max(n, 1), (stats[2], clip_frac)
+    assert abs(stats[3] - mean_r) <= 1e-5
+    g = grad if grad_slice is None else grad[grad_slice]
+    assert np.all((g == 0)[ok] == (g_ref == 0)[ok])
+    assert np.all(np.abs(g - g_ref)[ok] <= 1e-5 * np.abs(g_ref).max())
+    assert np.all(g[~m] == 0)
+    return undecided

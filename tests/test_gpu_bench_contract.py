@@ -58,3 +58,12 @@ def test_reference_arm_line():
     assert d["cpu_baseline"]["kind"] == "oracle" and d["cpu_baseline"]["value"] == d["value"]
     assert d["e2e"]["value"] == d["value"] and d["e2e"]["unit"] == d["unit"]
     assert d["e2e"]["h2d_bytes_per_step"] == 0 and d["e2e"]["d2h_bytes_per_step"] == 0
+
+
+def test_arms_emit_the_same_config():
+    """Both arms describe the same workload with the same config keys and
+    values, so their lines can be compared directly."""
+    a = run("--workload", "tiny", "--steps", "3", "--warmup", "3", "--no-cpu", "--no-e2e")
+    b = run("--impl", "reference", "--workload", "tiny", "--steps", "1", "--warmup", "1")
+    assert a["config"] == b["config"]
+    assert 0 < b["cpu_baseline"]["sample_fraction"] <= 1

@@ -5,7 +5,7 @@ import numpy as np
 import pytest
 import torch
 
-import oracle
+from tests.helpers import check_grpo
 
 pytestmark = pytest.mark.gpu
 
@@ -16,18 +16,6 @@ def hdl():
     __graft_entry__.build()
     import paper_2609_36864_gb300 as m
     return m
-
-
-def decided(lpn, lpo, eps_low=0.2, eps_high=0.28):
-    """Tokens whose clip decision both sides must take alike: the float32
-    ratio is more than 2 ulp from 1 - eps_low and 1 + eps_high (CUDA's expf
-    and numpy's float32 exp may round differently by up to 2 ulp, which can
-    flip the decision right at a bound)."""
-    r = np.exp(lpn.astype(np.float32) - lpo.astype(np.float32)).astype(np.float64)
-    ok = np.ones(len(r), dtype=bool)
-    for b in (np.float32(1.0) - np.float32(eps_low), np.float32(1.0) + np.float32(eps_high)):
-        ok &= np.abs(r - float(b)) > 2 * float(np.spacing(b))
-    return ok
 
 
 def make_batch(seed, n_groups, max_len):
@@ -55,22 +43,8 @@ def test_grpo_loss_matches_oracle(hdl, seed, n_groups, max_len):
     lpn, lpo, mask, toffs, R, goffs = make_batch(seed, n_groups, max_len)
     t = lambda x: torch.from_numpy(x).cuda()
     adv, grad, stats = hdl.hdl_grpo_loss(t(lpn), t(lpo), t(mask), t(toffs), t(R), t(goffs))
-    A_ref = oracle.group_advantages(R, goffs)
-    assert np.allclose(adv.cpu().numpy(), A_ref, rtol=0, atol=1e-6)
-    # the clip decision is taken in float32 on both sides (the kernel's
-    # precision); the values are compared against float64
-    loss, g_ref, (n, clip_frac, mean_r) = oracle.grpo_token_loss(
-        lpn, lpo, mask, toffs, adv.cpu().numpy().astype(np.float64), decide_in=np.float32)
-    st = stats.cpu().numpy()
-    assert st[1] == n
-    assert abs(st[0] - loss) <= 1e-5 * max(1.0, abs(loss))
-    assert abs(st[2] - clip_frac) <= 1e-6
-    assert abs(st[3] - mean_r) <= 1e-5
-    g = grad.cpu().numpy()
-    ok = decided(lpn, lpo)
-    assert np.all((g == 0)[ok] == (g_ref == 0)[ok])
-    assert np.all(np.abs(g - g_ref)[ok] <= 1e-5 * np.abs(g_ref).max())
-    assert np.all(g[mask == 0] == 0)
+    check_grpo(adv.cpu().numpy(), grad.cpu().numpy(), stats.cpu().numpy(), lpn, lpo, mask,
+               toffs, R, goffs)
 
 
 def test_grpo_paper_group(hdl):
@@ -97,7 +71,6 @@ def test_grpo_unaligned(hdl, shift, grad_off):
     offset (grad_off None: a fresh aligned buffer, or 2), which takes the
     scalar path."""
     lpn, lpo, mask, toffs, R, goffs = make_batch(10 + shift, 30, 200)
-    T = len(lpn)
     # `shift` leading tokens outside every trajectory, carrying no loss
     pad = lambda x, v: np.concatenate([np.full(shift, v, x.dtype), x])
     lpn2, lpo2, mask2 = pad(lpn, -1.0), pad(lpo, -1.0), pad(mask, 0)
@@ -110,14 +83,10 @@ def test_grpo_unaligned(hdl, shift, grad_off):
                                          torch.from_numpy(toffs2).cuda(),
                                          torch.from_numpy(R).cuda(),
                                          torch.from_numpy(goffs).cuda(), grad=grad)
-    loss, g_ref, (n, cf, mr) = oracle.grpo_token_loss(
-        lpn, lpo, mask, toffs, adv.cpu().numpy().astype(np.float64), decide_in=np.float32)
-    st = stats.cpu().numpy()
-    assert st[1] == n and abs(st[0] - loss) <= 1e-5 * max(1.0, abs(loss))
     g = grad.cpu().numpy()
     assert np.all(g[:shift] == 0)
-    ok = decided(lpn, lpo)
-    assert np.all(np.abs(g[shift:] - g_ref)[ok] <= 1e-5 * np.abs(g_ref).max())
+    check_grpo(adv.cpu().numpy(), g, stats.cpu().numpy(), lpn, lpo, mask, toffs, R, goffs,
+               grad_slice=slice(shift, None))
 
 
 def test_grpo_empty_inputs(hdl):

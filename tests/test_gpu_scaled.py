@@ -8,7 +8,7 @@ import pytest
 import torch
 
 import oracle
-from tests.test_gpu_grpo import decided
+from tests.helpers import check_grpo
 
 pytestmark = pytest.mark.gpu
 
@@ -57,18 +57,6 @@ def test_grpo_scaled(hdl):
     R = torch.rand(J, generator=g, device="cuda")
     goffs = torch.arange(0, J + 1, G, dtype=torch.int32, device="cuda")
     adv, grad, stats = hdl.hdl_grpo_loss(lpn, lpo, m, toffs, R, goffs)
-    lpn_h, lpo_h, m_h = lpn.cpu().numpy(), lpo.cpu().numpy(), m.cpu().numpy()
-    A_ref = oracle.group_advantages(R.cpu().numpy(), goffs.cpu().numpy())
-    assert np.allclose(adv.cpu().numpy(), A_ref, rtol=0, atol=1e-6)
-    loss, g_ref, (n, clip_frac, mean_r) = oracle.grpo_token_loss(
-        lpn_h, lpo_h, m_h, toffs.cpu().numpy(), adv.cpu().numpy().astype(np.float64),
-        decide_in=np.float32)
-    st = stats.cpu().numpy()
-    assert st[1] == n
-    assert abs(st[0] - loss) <= 1e-5 * max(1.0, abs(loss))
-    assert abs(st[2] - clip_frac) <= 1e-6
-    assert abs(st[3] - mean_r) <= 1e-5
-    gr = grad.cpu().numpy()
-    ok = decided(lpn_h, lpo_h)
-    assert np.all((gr == 0)[ok] == (g_ref == 0)[ok])
-    assert np.all(np.abs(gr - g_ref)[ok] <= 1e-5 * np.abs(g_ref).max())
+    check_grpo(adv.cpu().numpy(), grad.cpu().numpy(), stats.cpu().numpy(), lpn.cpu().numpy(),
+               lpo.cpu().numpy(), m.cpu().numpy(), toffs.cpu().numpy(), R.cpu().numpy(),
+               goffs.cpu().numpy())

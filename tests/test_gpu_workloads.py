@@ -5,7 +5,13 @@ with fp32 states (the tf32 path at a large shape).
 tiny and math: the oracle scores every token, so log-probs, scores and the
 end-to-end branch sets are compared in full.  code, agent and the sweep: the
 oracle scores sampled tokens one by one (first, last, random), and selection,
-allocation and masks are compared bit-exactly on the device's own scores."""
+allocation and masks are compared bit-exactly on the device's own scores; on
+top of that it scores whole roots (code: the first and the last; agent: the
+shortest, to bound the fp64 work; three sweep vocabularies: the last root),
+and on those every token's log-probs and |Delta| and the root's branch set
+(Section 3.2: the k highest-scoring valid positions) are compared with the
+oracle's -- branch sets equal except at positions whose oracle score is
+within 2e-3 of the root's k-th."""
 import dataclasses
 
 import numpy as np
@@ -94,6 +100,42 @@ def sampled_spec(which):
     return hdl_synth.SPECS[which]
 
 
+# whole roots scored by the oracle, per workload: "first_last", "shortest", "last"
+WHOLE_ROOTS = {"code": "first_last", "agent": "shortest", ("sweep", 32000, 1 << 20): "last",
+               ("sweep", 128256, 131072): "last", ("sweep", 256000, 262144): "last"}
+
+
+def whole_roots(wl, how):
+    R = wl.spec.n_roots
+    if how == "first_last":
+        return [0, R - 1]
+    if how == "shortest":
+        return [int(np.argmin(wl.lengths))]
+    return [R - 1]
+
+
+def check_whole_roots(wl, out, roots, W):
+    """Every token of each root in ``roots``, both contexts, against the
+    oracle, and the root's branch set against the oracle's on the oracle's
+    scores (the end-to-end band check)."""
+    offs = wl.root_offsets.cpu().numpy()
+    valid = wl.valid.cpu().numpy()
+    y_all = wl.targets.cpu().numpy()
+    k = wl.spec.k
+    for r in roots:
+        a, b = int(offs[r]), int(offs[r + 1])
+        r0 = oracle_logprobs(to_f64(wl.h_orig[a:b]), W, y_all[a:b], block=256)
+        r1 = oracle_logprobs(to_f64(wl.h_hind[a:b]), W, y_all[a:b], block=256)
+        what = f"{wl.spec.name} root {r} ({b - a} tokens)"
+        assert_logp_close(out["lp0"][a:b], r0, what + " orig")
+        assert_logp_close(out["lp1"][a:b], r1, what + " hind")
+        rd = oracle.hindsight_divergence(r1, r0)
+        err = np.abs(out["delta"][a:b] - rd)
+        assert np.all(err <= 2e-3 + 1e-3 * (np.abs(r0) + np.abs(r1))), (what, err.max())
+        check_selection_band(out["bp"][r:r + 1], out["ns"][r:r + 1], rd, valid[a:b],
+                             np.array([0, b - a]), k)
+
+
 @pytest.mark.parametrize("which", SAMPLED, ids=lambda w: w if isinstance(w, str) else
                          f"sweep_V{w[1]}_N{w[2]}")
 def test_workload_sampled(hdl, which):
@@ -106,9 +148,11 @@ def test_workload_sampled(hdl, which):
     y = wl.targets.cpu().numpy()[rows]
     r0 = oracle.target_logprobs(to_f64(wl.h_orig.index_select(0, idx)), W, y)
     r1 = oracle.target_logprobs(to_f64(wl.h_hind.index_select(0, idx)), W, y)
-    del W
     assert_logp_close(out["lp0"][rows], r0, spec.name + " orig")
     assert_logp_close(out["lp1"][rows], r1, spec.name + " hind")
+    if which in WHOLE_ROOTS:
+        check_whole_roots(wl, out, whole_roots(wl, WHOLE_ROOTS[which]), W)
+    del W
     check_downstream_exact(wl, out)
     # properties that hold at any size
     assert np.all(out["lp0"] <= 1e-5) and np.all(out["lp1"] <= 1e-5)

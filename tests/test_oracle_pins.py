@@ -453,11 +453,19 @@ def test_advantages():
 
 
 def check_grpo_loss(fn):
-    # hand cases of the asymmetric clip (eps 0.2 / 0.28), one token each
-    for r, A, want in ((1.5, 1.0, 1.28), (0.5, -1.0, -0.8), (0.5, 1.0, 0.5),
-                       (1.5, -1.0, -1.5), (1.1, 2.0, 2.2), (0.7, 1.0, 0.7)):
-        loss, grad, _ = fn([math.log(r)], [0.0], [1], [0, 1], [A])
+    # hand cases of the asymmetric clip (eps 0.2 / 0.28), one token each:
+    # (ratio, advantage, objective, gradient d loss / d logp_new, clipped?)
+    # -- the gradient is -r A where the unclipped term is the minimum (ties
+    # included: inside [0.8, 1.28] both terms are equal) and 0 where the
+    # clipped term is strictly smaller
+    for r, A, want, want_g, want_clip in (
+            (1.5, 1.0, 1.28, 0.0, 1), (0.5, -1.0, -0.8, 0.0, 1), (0.5, 1.0, 0.5, -0.5, 0),
+            (1.5, -1.0, -1.5, 1.5, 0), (1.1, 2.0, 2.2, -2.2, 0), (0.7, 1.0, 0.7, -0.7, 0),
+            (1.0, -3.0, -3.0, 3.0, 0)):
+        loss, grad, st = fn([math.log(r)], [0.0], [1], [0, 1], [A])
         assert abs(loss + want) < 1e-12, (r, A, loss)
+        assert abs(grad[0] - want_g) < 1e-12, (r, A, grad[0])
+        assert st[0] == 1 and st[1] == want_clip and abs(st[2] - r) < 1e-12, (r, A, st)
     # ratio 1: loss = -sum_j A_j L_j / sum_j L_j over masked tokens
     offs = [0, 3, 7, 8]
     mask = [1, 1, 0, 1, 1, 1, 1, 0]
@@ -525,6 +533,14 @@ def test_planted_mistakes_grpo():
 
     def no_clip(lpn, lpo, mask, offs, A):
         return O.grpo_token_loss(lpn, lpo, mask, offs, A, 1e9, 1e9)
-    for mutant in (symmetric_clip, sequence_mean, no_clip):
+
+    def ties_to_clipped(lpn, lpo, mask, offs, A):
+        # the gradient taken from the clipped term whenever it is not larger
+        loss, grad, st = O.grpo_token_loss(lpn, lpo, mask, offs, A)
+        r = np.exp(np.asarray(lpn, float) - np.asarray(lpo, float))
+        Aj = np.repeat(np.asarray(A, float), np.diff(offs))
+        tie = np.isclose(r * Aj, np.clip(r, 0.8, 1.28) * Aj, rtol=0, atol=0)
+        return loss, np.where(tie, 0.0, grad), st
+    for mutant in (symmetric_clip, sequence_mean, no_clip, ties_to_clipped):
         with pytest.raises(AssertionError):
             check_grpo_loss(mutant)
