@@ -85,12 +85,14 @@ HDL_API const char* hdl_status_string(hdl_status s);
  *   workspace       device scratch of at least
  *                   hdl_rescore_workspace_bytes(n_tokens, d, vocab, dt) bytes,
  *                   256-byte aligned, owned by the caller.  Its first word is
- *                   the device status word, cleared at the start of each call.
+ *                   the device status word; it and the merge counters after
+ *                   it are cleared (one memset) at the start of each call.
  *                   Two calls in flight at once must not share a workspace.
  * The [2N, V] logits are never written to memory: one persistent tensor-core
  * kernel walks the vocabulary tiles, keeps a running max and sum of
- * exponentials per row and picks out the target logit, then a small kernel
- * merges the per-vocabulary-chunk partial sums.
+ * exponentials per row and picks out the target logit; the same kernel
+ * merges the per-vocabulary-chunk partial sums of each 32 tokens as soon as
+ * the last of them is written (one memset + one kernel launch per call).
  */
 HDL_API size_t hdl_rescore_workspace_bytes(int64_t n_tokens, int32_t d, int32_t vocab,
                                    hdl_dtype dt);

@@ -9,9 +9,11 @@
 // the tile that holds it.
 //
 // Work unit = (M-tile of 128 rows of one context, vocabulary chunk of up to
-// 16 256-wide tiles).  Each unit writes one partial (max, sum) per row; a
-// second, small kernel merges the chunks, forms both log-probs, |Delta| and,
-// when asked, the entropies.  Units are rasterised in groups of 32 M-tiles x
+// 16 256-wide tiles).  Each unit writes one partial (max, sum) per row; the
+// epilogue warp that publishes the last partial of a 32-token slice (every
+// chunk, both contexts) merges the chunks of that slice, forming both
+// log-probs, |Delta| and, when asked, the entropies -- one launch for the
+// whole computation.  Units are rasterised in groups of 32 M-tiles x
 // the chunks, and the chunk is sized (see geometry) so that the H and W tiles
 // the ~150 concurrently running units touch stay in L2 -- W is then streamed
 // from DRAM once per group instead of once per M-tile.
@@ -106,6 +108,15 @@ struct RescoreArgs {
   int32_t target_offset;  // targets are shifted by this (vocabulary shards)
   uint32_t inject;     // test hook: bit 0 = the producer issues no copies
   uint64_t timeout_ns;
+  // Fused merge (null tile_done: the caller merges the partials itself).
+  // tile_done[4 * tt + q] counts the units that have published rows
+  // [128 tt + 32 q, +32) of either context; zeroed before the launch.
+  uint32_t* tile_done;
+  float* lp0;          // [N] log p^0
+  float* lp1;          // [N] log p^H
+  float* delta;        // [N] |Delta| or null
+  float* ent0;         // [N] entropy of the original context or null
+  float* ent1;         // [N] entropy of the hindsight context or null
 };
 
 struct Unit {
@@ -179,6 +190,44 @@ __device__ __forceinline__ void lse_fold_ent(const float (&x)[32], float& m2, fl
   s = fmaf(s, scale, (acc[0] + acc[1]) + (acc[2] + acc[3]));
   t = fmaf(t, scale, (acct[0] + acct[1]) + (acct[2] + acct[3]));
   m2 = m_new;
+}
+
+// Merge the per-chunk partials of both contexts of token t and write
+// log p^0, log p^H and |Delta| (Eq. div), and, when asked, the entropies
+// H = log Z - E_p[z] of both next-token distributions.  The partials were
+// written by other CTAs: they are read past L1.
+template <bool kEnt>
+__device__ __forceinline__ void merge_token(const RescoreArgs& a, int64_t t) {
+  const int64_t n = a.n_tokens, rows_total = 2 * n;
+  float lp[2], ent[2];
+#pragma unroll
+  for (int ctx = 0; ctx < 2; ++ctx) {
+    const int64_t g = ctx * n + t;
+    float M = -INFINITY;
+    for (int c = 0; c < a.num_chunks; ++c) M = fmaxf(M, __ldcg(a.part + c * rows_total + g).x);
+    float S = 0.f, T = 0.f;
+    for (int c = 0; c < a.num_chunks; ++c) {
+      const float2 p = __ldcg(a.part + c * rows_total + g);
+      const float sc = exp2f(p.x - M);
+      S += p.y * sc;
+      if constexpr (kEnt) T += __ldcg(a.part_t + c * rows_total + g) * sc;
+    }
+    const float lse = (M + log2f(S)) * kLn2;
+    lp[ctx] = __ldcg(a.zt + g) - lse;
+    ent[ctx] = lse - T / S;
+  }
+  const int32_t y = __ldg(a.targets + t);
+  if (y < 0 || y >= a.vocab) {
+    lp[0] = lp[1] = __int_as_float(0x7fc00000);
+    atomicOr(a.status, kStatusBadTarget);
+  }
+  a.lp0[t] = lp[0];
+  a.lp1[t] = lp[1];
+  if (a.delta) a.delta[t] = fabsf(lp[1] - lp[0]);
+  if constexpr (kEnt) {
+    if (a.ent0) a.ent0[t] = ent[0];
+    if (a.ent1) a.ent1[t] = ent[1];
+  }
 }
 
 // One persistent kernel for both contexts.  See Cfg for the two CTA
@@ -425,12 +474,29 @@ __global__ void __launch_bounds__(kThreads, 1)
             mbar_arrive(tempty_bar(buf));
         }
       }
-      if (ok && in_range) {
+      if (!ok) break;
+      if (in_range) {
         const int64_t rows_total = 2 * a.n_tokens;
         const int64_t g = w.ctx * a.n_tokens + row;
         a.part[static_cast<int64_t>(w.chunk) * rows_total + g] = make_float2(m2, s);
         if constexpr (kEnt) a.part_t[static_cast<int64_t>(w.chunk) * rows_total + g] = tz;
         if (found) a.zt[g] = zt;
+      }
+      // Fused merge: this warp's 32 rows are published; the warp that
+      // publishes the last of the 2 x num_chunks units of these rows (both
+      // contexts, every chunk) merges them.  Warp-local, so a warp that gave
+      // up above never leaves another one waiting.
+      const int tt = w.row0 / kBM;
+      if (a.tile_done != nullptr && tt < a.num_m_ctx) {
+        __threadfence();
+        __syncwarp();
+        uint32_t prev = 0;
+        if (lane == 0) prev = atomicAdd(a.tile_done + 4 * tt + q, 1u);
+        prev = __shfl_sync(0xffffffffu, prev, 0);
+        if (prev == 2u * static_cast<uint32_t>(a.num_chunks) - 1u) {
+          __threadfence();
+          if (in_range) merge_token<kEnt>(a, row);
+        }
       }
     }
   }
@@ -446,48 +512,6 @@ __global__ void __launch_bounds__(kThreads, 1)
       tmem_dealloc_pair(tmem_base, kTmemCols);
     else
       tmem_dealloc(tmem_base, kTmemCols);
-  }
-}
-
-// Merge the per-chunk partials of both contexts of token t and write
-// log p^0, log p^H and |Delta| (Eq. div), and, when asked, the entropies
-// H = log Z - E_p[z] of both next-token distributions.
-__global__ void __launch_bounds__(256)
-    rescore_merge_kernel(const float2* __restrict__ part, const float* __restrict__ part_t,
-                         const float* __restrict__ zt, const int32_t* __restrict__ targets,
-                         int64_t n, int32_t vocab, int32_t num_chunks, float* __restrict__ lp0,
-                         float* __restrict__ lp1, float* __restrict__ delta,
-                         float* __restrict__ ent0, float* __restrict__ ent1, uint32_t* status) {
-  const int64_t rows_total = 2 * n;
-  for (int64_t t = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x; t < n;
-       t += static_cast<int64_t>(gridDim.x) * blockDim.x) {
-    float lp[2], ent[2];
-#pragma unroll
-    for (int ctx = 0; ctx < 2; ++ctx) {
-      const int64_t g = ctx * n + t;
-      float M = -INFINITY;
-      for (int c = 0; c < num_chunks; ++c) M = fmaxf(M, part[c * rows_total + g].x);
-      float S = 0.f, T = 0.f;
-      for (int c = 0; c < num_chunks; ++c) {
-        const float2 p = part[c * rows_total + g];
-        const float sc = exp2f(p.x - M);
-        S += p.y * sc;
-        if (part_t) T += part_t[c * rows_total + g] * sc;
-      }
-      const float lse = (M + log2f(S)) * kLn2;
-      lp[ctx] = zt[g] - lse;
-      ent[ctx] = lse - T / S;
-    }
-    const int32_t y = targets[t];
-    if (y < 0 || y >= vocab) {
-      lp[0] = lp[1] = __int_as_float(0x7fc00000);
-      atomicOr(status, kStatusBadTarget);
-    }
-    lp0[t] = lp[0];
-    lp1[t] = lp[1];
-    if (delta) delta[t] = fabsf(lp[1] - lp[0]);
-    if (ent0) ent0[t] = ent[0];
-    if (ent1) ent1[t] = ent[1];
   }
 }
 
@@ -553,7 +577,7 @@ struct Geometry {
   int esize;
   int num_kb, num_m_ctx, num_m, num_vt, num_chunks, tiles_per_chunk;
   int64_t num_units;
-  size_t zt_off, part_off, part_t_off, total, total_ent;
+  size_t done_off, zt_off, part_off, part_t_off, total, total_ent;
 };
 
 // M-tiles per rasterisation group: HDL_GROUP_M (an even number in [2, 512])
@@ -612,7 +636,8 @@ Geometry geometry(int64_t n, int32_t d, int32_t vocab, hdl_dtype dt) {
   if (const int t = chunk_tiles_override(); t > 0 && t < g.tiles_per_chunk) g.tiles_per_chunk = t;
   g.num_chunks = static_cast<int>(ceil_div(g.num_vt, g.tiles_per_chunk));
   g.num_units = static_cast<int64_t>(g.num_m) * g.num_chunks;
-  g.zt_off = 256;
+  g.done_off = 256;   // after the status word: the fused merge's counters
+  g.zt_off = g.done_off + align_up(static_cast<size_t>(g.num_m_ctx) * 4 * sizeof(uint32_t), 256);
   g.part_off = g.zt_off + align_up(static_cast<size_t>(2 * n) * sizeof(float), 256);
   g.total = g.part_off + static_cast<size_t>(g.num_chunks) * static_cast<size_t>(2 * n) * sizeof(float2);
   g.part_t_off = align_up(g.total, 256);
@@ -817,9 +842,16 @@ extern "C" hdl_status hdl_rescore_ex(const void* h_orig, const void* h_hind,
   a.group_m = rescore_group_m();
   a.inject = o.fault_inject;
   a.timeout_ns = o.wait_timeout_ns ? o.wait_timeout_ns : kDefaultTimeoutNs;
+  a.tile_done = reinterpret_cast<uint32_t*>(ws + g.done_off);
+  a.lp0 = logp_orig;
+  a.lp1 = logp_hind;
+  a.delta = delta;
+  a.ent0 = o.entropy_orig;
+  a.ent1 = o.entropy_hind;
 
   cudaStream_t st = as_stream(cuda_stream);
-  if (cudaMemsetAsync(a.status, 0, sizeof(uint32_t), st) != cudaSuccess) return HDL_ERR_CUDA;
+  // the status word and the merge counters start at zero
+  if (cudaMemsetAsync(ws, 0, g.zt_off, st) != cudaSuccess) return HDL_ERR_CUDA;
 
   const int sms = current_sm_count();
   if (sms <= 0) return HDL_ERR_CUDA;
@@ -835,13 +867,6 @@ extern "C" hdl_status hdl_rescore_ex(const void* h_orig, const void* h_hind,
     ls = tf32 ? launch_rescore<true, 0, false>(tm_h0, tm_h1, tm_w, a, sms, st)
               : launch_rescore<false, 0, false>(tm_h0, tm_h1, tm_w, a, sms, st);
   if (ls != HDL_OK) return ls;
-  if (launch_status() != HDL_OK) return HDL_ERR_CUDA;
-
-  const int64_t mblocks = ceil_div(n_tokens, 256);
-  const int mgrid = static_cast<int>(mblocks < 8 * sms ? mblocks : 8 * sms);
-  rescore_merge_kernel<<<mgrid, 256, 0, st>>>(a.part, a.part_t, a.zt, targets, n_tokens, vocab,
-                                              g.num_chunks, logp_orig, logp_hind, delta,
-                                              o.entropy_orig, o.entropy_hind, a.status);
   return launch_status();
 }
 

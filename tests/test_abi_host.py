@@ -68,11 +68,13 @@ def _chunk_tiles(n, d, V, esize):
 
 
 def _ws_formula(n, d, V, esize=2):
-    """status (256 B) + target logits + per-(chunk, row) partials."""
+    """status (256 B) + merge counters (4 per 128-token tile) + target logits
+    + per-(chunk, row) partials."""
     cdiv = lambda a, b: -(-a // b)
     chunks = cdiv(cdiv(V, 256), _chunk_tiles(n, d, V, esize))
+    done = cdiv(cdiv(n, 128) * 4 * 4, 256) * 256
     zt = cdiv(2 * n * 4, 256) * 256
-    return 256 + zt + chunks * 2 * n * 8
+    return 256 + done + zt + chunks * 2 * n * 8
 
 
 @pytest.mark.parametrize("n,d,V", [(0, 64, 1), (1, 64, 1), (2048, 256, 4096),
