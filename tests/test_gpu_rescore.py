@@ -30,6 +30,10 @@ def run_and_check(hdl, wl, what):
     e1 = assert_logp_close(lp1.cpu().numpy(), r1, what + " hind")
     d = delta.cpu().numpy().astype(np.float64)
     assert np.array_equal(d, np.abs(lp1.cpu().numpy() - lp0.cpu().numpy()).astype(np.float64))
+    # and against the oracle's |Delta| (Eq. div), which inherits both contexts' errors
+    rd = np.abs(r1 - r0)
+    assert np.all(np.abs(d - rd) <= 2e-3 + 1e-3 * (np.abs(r0) + np.abs(r1))), \
+        (what, np.abs(d - rd).max())
     return max(e0, e1), r0, r1, d
 
 
