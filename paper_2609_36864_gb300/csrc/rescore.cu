@@ -52,7 +52,7 @@ constexpr int kBN = 256;             // vocabulary columns per tile
 constexpr int kRowBytes = 128;       // K bytes per stage (one 128-byte swizzle row)
 constexpr int kMaxTilesPerChunk = 16;  // up to 4096 vocabulary entries per unit
 constexpr int64_t kMinUnits = 1216;     // 8 x 152: chunks shrink until this many units
-constexpr double kL2Budget = 75e6;      // bytes of L2 the running units' tiles may use
+constexpr double kL2Budget = 70e6;      // bytes of L2 the running units' tiles may use
 constexpr int kPairsInFlight = 76;      // CTA pairs resident on 152 SMs
 #ifndef HDL_GROUP_M
 #define HDL_GROUP_M 32
@@ -615,12 +615,14 @@ Geometry geometry(int64_t n, int32_t d, int32_t vocab, hdl_dtype dt) {
   // The chunk: the largest power of two (<= 16 tiles) for which the tiles the
   // concurrently running units touch stay within kL2Budget of the 126 MB L2
   // -- the H tiles of one rasterisation group (group_m x 128 rows) plus the W
-  // tiles of the chunks in flight (one chunk per group_m / 2 running pairs,
-  // 76 pairs on 152 SMs).  Past that, W tiles are evicted before the group's
-  // last pairs use them: on the code-shaped workload 4-tile chunks read 90 GB
-  // from DRAM per launch instead of 156 GB and run 2.5 % faster, agent-shaped
-  // (d = 5120) 2-tile chunks 9 % faster, and working sets just above the
-  // budget (76-120 MB) were the slowest of all.
+  // tiles of the chunks in flight (one chunk per group_m / 2 running CTA
+  // pairs' worth of units, 76 pairs' worth on 152 SMs).  Past that, W tiles
+  // are evicted before the group's last units use them: on the code-shaped
+  // workload 4-tile chunks (64 MB) read 90 GB from DRAM per launch instead of
+  // 156 GB and run 2.5 % faster than 16-tile ones, agent-shaped (d = 5120)
+  // 2-tile chunks (67 MB) 9 % faster than 4-tile ones (92 MB), and at
+  // d = 4096 2-tile chunks (54 MB) up to 11 % faster than 4-tile ones
+  // (73 MB): working sets from about 70 MB up were the slowest.
   const double row = static_cast<double>(d) * g.esize;
   const int gm = rescore_group_m();
   const double h_bytes = gm * static_cast<double>(kBM) * row;

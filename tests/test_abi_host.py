@@ -56,11 +56,11 @@ def test_abi_version_and_names(L):
 def _chunk_tiles(n, d, V, esize):
     """Vocabulary tiles per chunk: from 16, halved while the H tiles of a group
     of 32 M-tiles plus the W tiles of the 76 / 16 chunks in flight exceed
-    75 MB, then while there are fewer than 1216 work units."""
+    70 MB, then while there are fewer than 1216 work units."""
     cdiv = lambda a, b: -(-a // b)
     num_m, nvt, tpc = 2 * cdiv(n, 128), cdiv(V, 256), 16
     row = d * esize
-    while tpc > 1 and 32 * 128 * row + (2 * 76 / 32) * tpc * 256 * row > 75e6:
+    while tpc > 1 and 32 * 128 * row + (2 * 76 / 32) * tpc * 256 * row > 70e6:
         tpc //= 2
     while tpc > 1 and num_m * cdiv(nvt, tpc) < 1216:
         tpc //= 2
