@@ -17,12 +17,9 @@
 // threshold.  The few candidates that beat the current k-th best (about
 // k ln(T/k) per root) are inserted one after the other (ballot + shift), or,
 // when many arrive together, by a bitonic sort of the warp's 32 candidates
-// and a bitonic merge with the list.  Few roots: 16 warps per root; the
-// partial lists of a root's warps are merged pairwise, a bitonic merge per
-// level.  Many roots (at least two per resident CTA): runs of roots, one run
-// per CTA, whose positions its 8 warps split evenly across root boundaries
-// (select_run_kernel); in between, and for the greedy spacing rule, S warps
-// per root (usually 1) in a persistent grid.
+// and a bitonic merge with the list.  Many roots: S warps per root (usually
+// 1) in a persistent grid; few roots: 16 warps per root; the partial lists
+// of a root's warps are merged pairwise, a bitonic merge per level.
 // Spacing rule (Section 4.4; min_gap > 0, |t - a| < min_gap counts as too
 // close):
 //   drop-lower (gap_mode 1): the plain top-k above, then the root's warp walks
@@ -425,34 +422,6 @@ __device__ __forceinline__ bool collect(WarpTopK& w, uint64_t (*lists)[32], cons
 
 enum SelectMode : int { kPlain = 0, kDropLower = 1, kGreedy = 2 };
 
-// Root r's result from its finished list (lanes 0..n-1, best first; 0 in the
-// other lanes), after the drop-lower spacing rule when asked: positions,
-// scores (-1 / NaN padding) and the count.
-template <int kMode>
-__device__ __forceinline__ void finish_root(WarpTopK& w, int64_t r, int64_t start, int k,
-                                            int32_t min_gap, const float* delta,
-                                            int32_t* branch_pos, int32_t* n_selected,
-                                            float* branch_delta, int lane) {
-  int n = __popc(__ballot_sync(0xffffffffu, w.mine != 0ull));
-  if constexpr (kMode == kDropLower) {
-    if (n > 1) drop_close(w, n, min_gap, lane);
-  }
-  if (lane < k) {
-    const int64_t o = r * k + lane;
-    if (lane < n) {
-      const int64_t t = key_pos(w.mine);
-      branch_pos[o] = static_cast<int32_t>(t);
-      // the key holds the absolute position minus the root start, mod 2^32
-      if (branch_delta)
-        branch_delta[o] = delta[static_cast<uint32_t>(start) + static_cast<uint32_t>(t)];
-    } else {
-      branch_pos[o] = -1;
-      if (branch_delta) branch_delta[o] = __int_as_float(0x7fc00000);
-    }
-  }
-  if (lane == 0) n_selected[r] = n;
-}
-
 // kMode: plain top-k; drop-lower spacing applied to the finished list; or
 // greedy spacing -- passes that each collect the kMaxK best positions far
 // enough from every point accepted so far and walk them in rank order,
@@ -488,8 +457,24 @@ __global__ void __launch_bounds__(32 * TopkShape<S>::kWarps, TopkShape<S>::kMinB
       if (!collect<S, kVec>(w, lists, delta, valid, start, a0, a1, k, lane, warp, grp, ws, phase,
                             AnyPos{}))
         continue;
-      finish_root<kMode>(w, r, start, k, min_gap, delta, branch_pos, n_selected, branch_delta,
-                         lane);
+      int n = __popc(__ballot_sync(0xffffffffu, w.mine != 0ull));
+      if constexpr (kMode == kDropLower) {
+        if (n > 1) drop_close(w, n, min_gap, lane);
+      }
+      if (lane < k) {
+        const int64_t o = r * k + lane;
+        if (lane < n) {
+          const int64_t t = key_pos(w.mine);
+          branch_pos[o] = static_cast<int32_t>(t);
+          // the key holds the absolute position minus the root start, mod 2^32
+          if (branch_delta)
+            branch_delta[o] = delta[static_cast<uint32_t>(start) + static_cast<uint32_t>(t)];
+        } else {
+          branch_pos[o] = -1;
+          if (branch_delta) branch_delta[o] = __int_as_float(0x7fc00000);
+        }
+      }
+      if (lane == 0) n_selected[r] = n;
     } else {
       int32_t* acc = accepted[grp];
       FarFromAccepted far{acc, 0, min_gap};
@@ -539,130 +524,6 @@ __global__ void __launch_bounds__(32 * TopkShape<S>::kWarps, TopkShape<S>::kMinB
   }
 }
 
-// Many roots (plain top-k and drop-lower): each CTA takes a contiguous run of
-// roots (split by count) and its 8 warps split the run's positions evenly,
-// crossing root boundaries, so that every resident warp streams for the whole
-// launch instead of a last, partly filled round of one-warp-per-root work.  A
-// root inside one warp's range is finished by that warp.  A root cut by a
-// warp boundary leaves the exact top-k list of each of its pieces in shared
-// memory; after one barrier a warp merges them (the k best of a root are
-// among the k best of its pieces) and finishes the root.  A run whose offsets
-// are not monotone is done one warp per root, as the per-root kernel does.
-constexpr int kRunWarps = 8;
-constexpr int kMaxRun = 32;   // roots per CTA at most (the launch sizes the grid so)
-
-template <bool kVec, int kMode>
-__global__ void __launch_bounds__(32 * kRunWarps, 4)
-    select_run_kernel(const float* __restrict__ delta, const uint8_t* __restrict__ valid,
-                      int64_t n_tokens, const int64_t* __restrict__ root_offsets,
-                      int32_t n_roots, int32_t k, int32_t lo, int32_t hi, int32_t min_gap,
-                      int32_t phase, int32_t* __restrict__ branch_pos,
-                      int32_t* __restrict__ n_selected, float* __restrict__ branch_delta) {
-  __shared__ int64_t st[kMaxRun + 1];            // the run's root offsets
-  __shared__ int64_t bnd[kRunWarps + 1];         // warp v streams [bnd[v], bnd[v+1])
-  __shared__ uint64_t pieces[kRunWarps][2][kMaxK];  // lists of the warp's first / last cut root
-  __shared__ int mono;
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  const int64_t r0 = static_cast<int64_t>(blockIdx.x) * n_roots / gridDim.x;
-  const int64_t r1 = static_cast<int64_t>(blockIdx.x + 1) * n_roots / gridDim.x;
-  const int nr = static_cast<int>(r1 - r0);
-  if (static_cast<int>(threadIdx.x) <= nr) st[threadIdx.x] = root_offsets[r0 + threadIdx.x];
-  __syncthreads();
-  auto clampn = [&](int64_t x) { return x < 0 ? int64_t{0} : (x > n_tokens ? n_tokens : x); };
-  if (warp == 0) {
-    bool ok = true;
-    for (int i = lane; i < nr; i += 32) ok = ok && st[i] <= st[i + 1];
-    ok = __all_sync(0xffffffffu, ok);
-    if (lane == 0) {
-      mono = ok;
-      const int64_t S = clampn(st[0]), E = clampn(st[nr]);
-      bnd[0] = S;
-      bnd[kRunWarps] = E;
-      for (int v = 1; v < kRunWarps; ++v) {
-        // even shares, each starting on a 128-byte line of the scores
-        int64_t b = S + (E - S) * v / kRunWarps;
-        b = ((b + phase) & ~int64_t{31}) - phase;
-        bnd[v] = b < bnd[v - 1] ? bnd[v - 1] : (b > E ? E : b);
-      }
-    }
-  }
-  __syncthreads();
-  // root j's candidate window [a0, a1), as the per-root kernel forms it
-  auto window = [&](int j, int64_t& a0, int64_t& a1) {
-    const int64_t start = st[j], end = st[j + 1];
-    const int64_t T = end > start ? end - start : 0;
-    const int64_t w_lo = lo > 0 ? lo : 0;
-    const int64_t w_hi = hi <= 0 ? T : (hi < T ? hi : T);
-    a0 = start + w_lo;
-    a1 = start + w_hi;
-    if (a0 < 0) a0 = 0;
-    if (a1 > n_tokens) a1 = n_tokens;
-  };
-  WarpTopK w;
-  if (!mono) {
-    for (int j = warp; j < nr; j += kRunWarps) {
-      int64_t a0, a1;
-      window(j, a0, a1);
-      w = WarpTopK{0ull, 0ull, -INFINITY, -INFINITY};
-      if (a1 > a0) stream_range<kVec>(w, delta, valid, st[j], a0, a1, k, lane, phase, AnyPos{});
-      finish_root<kMode>(w, r0 + j, st[j], k, min_gap, delta, branch_pos, n_selected,
-                         branch_delta, lane);
-    }
-    return;
-  }
-  // the warp whose range holds position p (S <= p < E): the last v with bnd[v] <= p
-  // (never an empty range: an empty one shares its bound with the next)
-  auto owner = [&](int64_t p) {
-    int v = kRunWarps - 1;
-    while (v > 0 && bnd[v] > p) --v;
-    return v;
-  };
-  // streaming: the pieces of the roots that meet this warp's range
-  const int64_t A = bnd[warp], B = bnd[warp + 1];
-  for (int j = 0; j < nr && A < B; ++j) {
-    const int64_t s0 = clampn(st[j]), e0 = clampn(st[j + 1]);
-    if (s0 >= e0 || e0 <= A || s0 >= B) continue;
-    int64_t a0, a1;
-    window(j, a0, a1);
-    if (a0 < A) a0 = A;
-    if (a1 > B) a1 = B;
-    w = WarpTopK{0ull, 0ull, -INFINITY, -INFINITY};
-    if (a1 > a0) stream_range<kVec>(w, delta, valid, st[j], a0, a1, k, lane, phase, AnyPos{});
-    if (s0 >= A && e0 <= B) {
-      finish_root<kMode>(w, r0 + j, st[j], k, min_gap, delta, branch_pos, n_selected,
-                         branch_delta, lane);
-    } else if (lane < kMaxK) {
-      if (s0 < A) pieces[warp][0][lane] = w.mine;   // began in an earlier warp's range
-      if (e0 > B) pieces[warp][1][lane] = w.mine;   // goes on in a later warp's range
-    }
-  }
-  __syncthreads();
-  // cut and empty roots, round robin over the warps
-  int turn = 0;
-  for (int j = 0; j < nr; ++j) {
-    const int64_t s0 = clampn(st[j]), e0 = clampn(st[j + 1]);
-    int wf = 0, wl = 0;
-    if (s0 < e0) {
-      wf = owner(s0);
-      wl = owner(e0 - 1);
-      if (wf == wl) continue;   // finished while streaming
-    }
-    if (turn++ % kRunWarps != warp) continue;
-    uint64_t acc = 0ull;
-    if (s0 < e0) {
-      acc = lane < kMaxK ? pieces[wf][1][lane] : 0ull;
-      for (int v = wf + 1; v <= wl; ++v) {
-        if (bnd[v] == bnd[v + 1]) continue;   // an empty range holds no piece
-        const uint64_t m = bitonic_merge16(acc, pieces[v][0][(31 - lane) & 15], lane);
-        acc = lane < k ? m : 0ull;
-      }
-    }
-    w.mine = acc;
-    finish_root<kMode>(w, r0 + j, st[j], k, min_gap, delta, branch_pos, n_selected,
-                       branch_delta, lane);
-  }
-}
-
 // HDL_SELECT_SPLIT (1, 2, 4 or 8) fixes the warps per root of the many-roots
 // mode, for tests and tuning; results do not depend on it.
 int select_split_override() {
@@ -707,41 +568,9 @@ hdl_status launch_topk_s(const SelectArgs& a, int grid, cudaStream_t st) {
 // and occupancy; neither deeper register prefetch nor a shared-memory ring
 // filled by bulk copies made it faster.)  kMode selects the spacing rule,
 // with min_gap = a.gap.
-// Runs of roots for the many-roots case: one wave of resident CTAs when that
-// gives each at most kMaxRun roots, else enough CTAs for kMaxRun each.
-template <bool kVec, int kMode>
-hdl_status launch_run(const SelectArgs& a, int64_t ctas, cudaStream_t st) {
-  const int64_t need = (int64_t{a.n_roots} + kMaxRun - 1) / kMaxRun;
-  const int64_t grid = ctas > need ? ctas : need;
-  select_run_kernel<kVec, kMode><<<static_cast<unsigned>(grid), 32 * kRunWarps, 0, st>>>(
-      a.delta, a.valid, a.n_tokens, a.offs, a.n_roots, a.k, a.lo, a.hi, a.gap, a.phase, a.bp,
-      a.ns, a.bd);
-  return launch_status();
-}
-
-// HDL_SELECT_RUNS = 0 turns the runs of roots off (the per-root kernel takes
-// every case), for tests and tuning; results do not depend on it.
-bool select_runs_enabled() {
-  static const bool v = [] {
-    const char* e = std::getenv("HDL_SELECT_RUNS");
-    return !(e && e[0] == '0' && e[1] == '\0');
-  }();
-  return v;
-}
-
 template <bool kVec, int kMode>
 hdl_status launch_topk(const SelectArgs& a, int sms, cudaStream_t st) {
   if (a.n_roots < 2 * sms) return launch_topk_s<16, kVec, kMode>(a, a.n_roots, st);
-  if constexpr (kMode != kGreedy) {
-    // at least two roots per resident CTA: runs of roots, one wave
-    int run_per_sm = 0;
-    if (select_runs_enabled() && select_split_override() == 0 &&
-        cudaOccupancyMaxActiveBlocksPerMultiprocessor(&run_per_sm,
-                                                      select_run_kernel<kVec, kMode>,
-                                                      32 * kRunWarps, 0) == cudaSuccess &&
-        run_per_sm > 0 && int64_t{a.n_roots} >= 2 * int64_t{run_per_sm} * sms)
-      return launch_run<kVec, kMode>(a, int64_t{run_per_sm} * sms, st);
-  }
   int per_sm = 0;
   if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, select_topk_kernel<1, kVec, kMode>,
                                                     256, 0) != cudaSuccess || per_sm <= 0)

@@ -356,32 +356,9 @@ def test_select_randomized(hdl):
         assert_select_equal(hdl, delta, valid if case % 5 else None, offs, k, lo=lo, hi=hi)
 
 
-_RUNS_SCRIPT = r"""
-import sys
-import numpy as np
-import torch
-sys.path.insert(0, sys.argv[1])
-import paper_2609_36864_gb300 as hdl
-data = np.load(sys.argv[2])
-d = torch.from_numpy(data["delta"]).cuda()
-v = torch.from_numpy(data["valid"]).cuda()
-o = torch.from_numpy(data["offs"]).cuda()
-out = {}
-for k in (1, 8, 16):
-    for lo, hi in ((0, 0), (3, 40)):
-        bp, ns, bd = hdl.hdl_select_branches(d, v, o, k, lo=lo, hi=hi)
-        out[f"bp{k}_{lo}"], out[f"ns{k}_{lo}"], out[f"bd{k}_{lo}"] = (
-            bp.cpu().numpy(), ns.cpu().numpy(), bd.cpu().numpy())
-    bp, ns, bd = hdl.hdl_select_branches(d, v, o, k, min_gap=5, gap_mode=1)
-    out[f"bp{k}_drop"], out[f"ns{k}_drop"] = bp.cpu().numpy(), ns.cpu().numpy()
-np.savez(sys.argv[3], **out)
-"""
-
-
 def runs_case(seed, n_roots=1700):
-    """Many roots (at least two per resident CTA of the runs-of-roots path):
-    mostly short, some empty, and every 97th one long enough to span all the
-    warps of its CTA's range."""
+    """Many roots (more than the resident warps): mostly short, some empty,
+    and every 97th one long (3000-12000 positions)."""
     rng = np.random.default_rng(seed)
     lengths = rng.integers(0, 120, size=n_roots)
     lengths[::13] = 0
@@ -389,44 +366,12 @@ def runs_case(seed, n_roots=1700):
     return make_roots(list(lengths), seed + 1, tie_levels=30, nan_frac=0.01)
 
 
-def test_select_runs_of_roots(hdl, tmp_path):
-    """The runs-of-roots path (each CTA's warps split its run's positions
-    evenly, crossing root boundaries; roots cut by a warp boundary are merged
-    from their pieces): bit-exact against the oracle and against the
-    per-root kernel (HDL_SELECT_RUNS=0), with windows, every k and the
-    drop-lower spacing rule."""
-    delta, valid, offs = runs_case(31)
-    inp = tmp_path / "in.npz"
-    np.savez(inp, delta=delta, valid=valid, offs=offs)
-    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
-    got = {}
-    for runs in ("1", "0"):
-        outp = tmp_path / f"out{runs}.npz"
-        subprocess.run([sys.executable, "-c", _RUNS_SCRIPT, root, str(inp), str(outp)],
-                       env=dict(os.environ, HDL_SELECT_RUNS=runs), check=True, timeout=300)
-        got[runs] = np.load(outp)
-    for key in got["1"].files:
-        assert np.array_equal(got["1"][key], got["0"][key], equal_nan=True), key
-    for k in (1, 8, 16):
-        for lo, hi in ((0, 0), (3, 40)):
-            pos, nsel, val = oracle.select_branches(delta.astype(np.float64), valid, offs, k,
-                                                    lo=lo, hi=hi)
-            assert np.array_equal(got["1"][f"ns{k}_{lo}"], nsel)
-            assert np.array_equal(got["1"][f"bp{k}_{lo}"], pos)
-            assert np.array_equal(got["1"][f"bd{k}_{lo}"].astype(np.float64), val,
-                                  equal_nan=True)
-        pos, nsel, _ = oracle.select_branches(delta.astype(np.float64), valid, offs, k,
-                                              min_gap=5, gap_mode=1)
-        assert np.array_equal(got["1"][f"ns{k}_drop"], nsel)
-        assert np.array_equal(got["1"][f"bp{k}_drop"], pos)
-
-
 @pytest.mark.parametrize("d_off,v_off", OFFSETS)
-def test_select_runs_unaligned_and_nonmonotone(hdl, d_off, v_off):
-    """Runs of roots on buffers off their alignment (the phase-shifted vector
-    path and the element-by-element one), and with a few roots whose end
-    precedes their start (their run is done one warp per root): the oracle's
-    result bit for bit."""
+def test_select_many_roots_unaligned_and_nonmonotone(hdl, d_off, v_off):
+    """1700 ragged roots (short, empty and long ones) on buffers off their
+    alignment (the phase-shifted vector path and the element-by-element one),
+    with a few roots whose end precedes their start: the oracle's result bit
+    for bit."""
     delta, valid, offs = runs_case(40 + d_off + 4 * v_off)
     offs = offs.copy()
     for r in (7, 600, 1333):                      # end before start: an empty root
