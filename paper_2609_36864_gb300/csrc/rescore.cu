@@ -494,6 +494,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (lane == 0) prev = atomicAdd(a.tile_done + 4 * tt + q, 1u);
         prev = __shfl_sync(0xffffffffu, prev, 0);
         if (prev == 2u * static_cast<uint32_t>(a.num_chunks) - 1u) {
+          // lane 0 saw every unit counted: order the lanes' reads after it
+          __syncwarp();
           __threadfence();
           if (in_range) merge_token<kEnt>(a, row);
         }

@@ -102,7 +102,17 @@ def check_grpo(adv, grad, stats, lpn, lpo, mask, toffs, rewards, goffs, grad_sli
     assert abs(stats[2] - clip_frac) <= 1e-6 + undecided / max(n, 1), (stats[2], clip_frac)
     assert abs(stats[3] - mean_r) <= 1e-5
     g = grad if grad_slice is None else grad[grad_slice]
+    tol = 1e-5 * np.abs(g_ref).max() if g_ref.size else 0.0
     assert np.all((g == 0)[ok] == (g_ref == 0)[ok])
-    assert np.all(np.abs(g - g_ref)[ok] <= 1e-5 * np.abs(g_ref).max())
+    assert np.all(np.abs(g - g_ref)[ok] <= tol)
     assert np.all(g[~m] == 0)
+    # near a bound either term may be the minimum: the gradient there is the
+    # unclipped one, -r A / n, or 0, and nothing else
+    amb = m & ~ok
+    if amb.any():
+        r = np.exp(np.asarray(lpn, np.float64) - np.asarray(lpo, np.float64))
+        A = np.repeat(A_ref, np.diff(np.asarray(toffs, np.int64)))
+        unclipped = -r * A / n
+        dev = np.minimum(np.abs(g - unclipped), np.abs(g))[amb]
+        assert np.all(dev <= tol), dev.max()
     return undecided
