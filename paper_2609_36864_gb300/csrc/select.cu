@@ -216,8 +216,9 @@ __device__ __forceinline__ void load_batch(Batch& b, const float* delta, const u
 // Otherwise the lanes' passing valid candidates are offered in rounds, each
 // lane its next one per round, until no lane has any left.
 template <class F>
-__device__ __forceinline__ void offer_batch(WarpTopK& w, const Batch& b, int32_t q,
-                                            int32_t start, int k, int lane, const F& f) {
+__device__ __forceinline__ void offer_batch(WarpTopK& w, const Batch& b, const float* delta,
+                                            int32_t q, int32_t start, int k, int lane,
+                                            const F& f) {
   float mx = -INFINITY;   // fmaxf ignores NaN scores
 #pragma unroll
   for (int i = 0; i < kBatch; ++i)
@@ -236,15 +237,11 @@ __device__ __forceinline__ void offer_batch(WarpTopK& w, const Batch& b, int32_t
   while (__any_sync(0xffffffffu, pass != 0)) {
     const int j = pass ? __ffs(pass) - 1 : -1;
     pass &= pass - 1u;
-    float sj = -INFINITY;
-#pragma unroll
-    for (int i = 0; i < kBatch; ++i) {
-      sj = j == 4 * i ? b.d[i].x : sj;
-      sj = j == 4 * i + 1 ? b.d[i].y : sj;
-      sj = j == 4 * i + 2 ? b.d[i].z : sj;
-      sj = j == 4 * i + 3 ? b.d[i].w : sj;
-    }
-    const int32_t t = q + 4 * (32 * (j >> 2) + lane) + (j & 3) - start;
+    // the candidate's score, read again from the batch just loaded (a cache
+    // hit; cheaper in instructions than selecting it among 16 registers)
+    const int32_t p = q + 4 * (32 * (j >> 2) + lane) + (j & 3);
+    const float sj = j >= 0 ? delta[p] : -INFINITY;
+    const int32_t t = p - start;
     wtk_offer_key(w, j >= 0 && sj >= w.tau_s && f.ok(t) ? make_key(sj, t) : 0ull, k, lane);
   }
 }
@@ -334,7 +331,7 @@ __device__ __forceinline__ void stream_range(WarpTopK& w, const float* delta, co
     else
       load_batch<false>(x, delta, valid, q, body, lane);
     if (q == h) set_floor(w, x, q, start, k, lane, f);
-    offer_batch(w, x, q, start, k, lane, f);
+    offer_batch(w, x, delta, q, start, k, lane, f);
   }
   // scalar head and tail (at most 3 positions each)
   const int32_t p = lane < 4 ? a0 + lane : body + (lane - 4);
