@@ -67,3 +67,14 @@ def test_arms_emit_the_same_config():
     b = run("--impl", "reference", "--workload", "tiny", "--steps", "1", "--warmup", "1")
     assert a["config"] == b["config"]
     assert 0 < b["cpu_baseline"]["sample_fraction"] <= 1
+
+
+def test_graph_replay_line():
+    """--graph: the kernel-only steps and the end-to-end steps (input copies,
+    the four calls, result copies) are replayed from CUDA graphs; the line
+    keeps every key."""
+    d = run("--workload", "tiny", "--steps", "3", "--warmup", "3", "--no-cpu", "--graph")
+    assert d["config"]["launch"].startswith("CUDA graph")
+    e = d["e2e"]
+    assert num(e["value"]) and e["value"] > 0 and "graph" in e["overlap"]
+    assert e["h2d_bytes_per_step"] > 0 and e["d2h_bytes_per_step"] > 0
