@@ -362,9 +362,11 @@ def cpu_oracle_parity(wl, lp0, lp1, count: int = 40, seed: int = 0):
             "tolerance": "1e-3 + 1e-3 |ref|", "within": within}
 
 
-# The other workloads the tensor-peak target is stated on, timed after the
-# default one (kernel only: the fused re-scoring call, inputs resident).
-EXTRA_WORKLOADS = ("agent", "sweep_V32000_N262144", "sweep_V256000_N262144")
+# The other large workloads, timed after the default one (kernel only: the
+# fused re-scoring call, inputs resident and larger than twice the L2, so the
+# steps run back to back): the agent-shaped one and the two largest sweep
+# points, on which the tensor-peak target is stated, and the math-shaped one.
+EXTRA_WORKLOADS = ("agent", "sweep_V32000_N262144", "sweep_V256000_N262144", "math")
 
 
 def time_extra_workloads(hdl, args, local, check: bool):
@@ -384,8 +386,14 @@ def time_extra_workloads(hdl, args, local, check: bool):
                                        delta, ws, stream=stream)
         for _ in range(2):
             call()
+        # enough steps for a timed region of at least half a second (clock samples)
+        t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        t0.record(stream)
+        call()
+        t1.record(stream)
         torch.cuda.synchronize()
-        steps = args.extra_steps
+        one_ms = max(t0.elapsed_time(t1), 1e-3)
+        steps = max(args.extra_steps, min(200, int(np.ceil(500.0 / one_ms))))
         ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
               for _ in range(steps)]
         clocks = ClockSampler(local)
