@@ -8,7 +8,9 @@
  * Conventions shared by every entry point
  *   - Array arguments are DEVICE pointers unless stated otherwise.  The caller
  *     owns every buffer; the library allocates no device memory and keeps no
- *     per-call state between calls.
+ *     per-call state between calls.  (The one exception is the module's own
+ *     static scratch array, which only hdl_rescore_noalloc uses; it is loaded
+ *     with the library on each device, see there.)
  *   - Calls are asynchronous on `cuda_stream` (a cudaStream_t; NULL = the
  *     legacy default stream).  Argument errors are detected on the host and
  *     returned before anything is launched.  A failed launch returns
