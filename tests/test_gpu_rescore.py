@@ -318,3 +318,29 @@ def test_rescore_wide_hidden(hdl, d, dt):
     y = wl.targets.cpu().numpy()
     assert_logp_close(lp0.cpu().numpy(), oracle_logprobs(to_f64(wl.h_orig), W, y), "wide orig")
     assert_logp_close(lp1.cpu().numpy(), oracle_logprobs(to_f64(wl.h_hind), W, y), "wide hind")
+
+
+def test_rescore_randomized(hdl):
+    """24 seeded random shapes (tokens 1-700, d a multiple of 64 up to 1024,
+    vocabularies 1-10000, bf16 and fp32 states): log-probs, |Delta| and both
+    entropies against the oracle element by element."""
+    import oracle
+    rng = np.random.default_rng(77)
+    for case in range(24):
+        n = int(rng.integers(1, 701))
+        d = 64 * int(rng.integers(1, 17))
+        V = int(rng.integers(1, 10001))
+        dt = "f32" if case % 4 == 3 else "bf16"
+        spec = hdl_synth.small_spec(f"rand{case}", n_roots=1, t_lo=n, t_hi=n, d=d, vocab=V,
+                                    dtype=dt, seed=1000 + case)
+        wl = hdl_synth.generate(spec, device="cuda")
+        err, r0, r1, dl = run_and_check(hdl, wl, f"random case {case} {(n, d, V, dt)}")
+        if case % 3 == 0:
+            lp0, lp1, de, e0, e1, ws = hdl.hdl_rescore_ex(wl.h_orig, wl.h_hind, wl.w, wl.targets,
+                                                          want_entropy_hind=True)
+            assert hdl.hdl_device_status(ws)[0] == hdl.HDL_OK
+            W = to_f64(wl.w)
+            assert_logp_close(e0.cpu().numpy(), oracle.next_token_entropy(to_f64(wl.h_orig), W),
+                              f"random case {case} entropy orig")
+            assert_logp_close(e1.cpu().numpy(), oracle.next_token_entropy(to_f64(wl.h_hind), W),
+                              f"random case {case} entropy hind")

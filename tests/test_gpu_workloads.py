@@ -174,3 +174,35 @@ def test_workload_entropy_selector(hdl, name):
     assert_logp_close(e0.cpu().numpy(), ref, name + " entropy")
     check_selection_band(bp.cpu().numpy(), ns.cpu().numpy(), ref, wl.valid.cpu().numpy(),
                          wl.root_offsets.cpu().numpy(), wl.spec.k)
+
+
+def test_random_small_workloads_end_to_end(hdl):
+    """12 seeded random small workloads through the whole path (re-scoring,
+    selection, allocation, masks): every token's log-probs and |Delta|
+    against the oracle, branch sets within the band of the root's k-th
+    oracle score (Section 3.2), and selection / allocation / masks bit-exact
+    on the device's scores."""
+    rng = np.random.default_rng(4242)
+    for case in range(12):
+        T_lo = int(rng.integers(1, 400))
+        spec = hdl_synth.small_spec(
+            f"e2e{case}", n_roots=int(rng.integers(1, 13)), t_lo=T_lo,
+            t_hi=T_lo + int(rng.integers(0, 1200)), d=64 * int(rng.integers(1, 9)),
+            vocab=int(rng.integers(50, 20001)), dtype="f32" if case % 5 == 4 else "bf16",
+            k=int(rng.integers(1, 17)), pert_frac=float(rng.choice([0.01, 0.05, 0.2])),
+            pert_mode=str(rng.choice(["uniform", "spans", "valid"])),
+            invalid_frac=float(rng.choice([0.0, 0.2])),
+            conts_per_root=int(rng.integers(1, 9)), seed=500 + case)
+        wl = hdl_synth.generate(spec, device="cuda")
+        out = run_path(hdl, wl)
+        W = to_f64(wl.w)
+        y = wl.targets.cpu().numpy()
+        r0 = oracle_logprobs(to_f64(wl.h_orig), W, y)
+        r1 = oracle_logprobs(to_f64(wl.h_hind), W, y)
+        assert_logp_close(out["lp0"], r0, f"{spec.name} orig")
+        assert_logp_close(out["lp1"], r1, f"{spec.name} hind")
+        rd = oracle.hindsight_divergence(r1, r0)
+        assert np.all(np.abs(out["delta"] - rd) <= 2e-3 + 1e-3 * (np.abs(r0) + np.abs(r1)))
+        check_selection_band(out["bp"], out["ns"], rd, wl.valid.cpu().numpy(),
+                             wl.root_offsets.cpu().numpy(), spec.k)
+        check_downstream_exact(wl, out)
