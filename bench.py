@@ -45,6 +45,10 @@ def parse():
                         "(math_f32) gives fp32 hidden states and LM head (tf32 products)")
     p.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
     p.add_argument("--no-e2e", action="store_true")
+    p.add_argument("--shards", type=int, default=0,
+                   help="re-score through the vocabulary-parallel entry points on this one GPU: "
+                        "W cut into this many row shards (at 256-row tile boundaries), one "
+                        "hdl_rescore_shard call per shard, then hdl_merge_vocab_shards")
     p.add_argument("--graph", action="store_true",
                    help="capture one step in a CUDA graph and time its replays "
                         "(for launch-bound workloads such as tiny)")
@@ -122,9 +126,10 @@ def input_bytes(wl) -> int:
     return sum(t.numel() * t.element_size() for t in (wl.h_orig, wl.h_hind, wl.w))
 
 
-def workload_config(spec, wl, graph: bool) -> dict:
+def workload_config(spec, wl, graph: bool, shards: int = 0) -> dict:
     """The ``config`` of the JSON line, identical for both arms: the workload,
-    its sizes and how L2 is handled between timed steps."""
+    its sizes, how L2 is handled between timed steps and, when the LM head is
+    cut into vocabulary shards, their number."""
     in_bytes = input_bytes(wl)
     l2 = (f"inputs larger than L2 ({in_bytes / 2**30:.2f} GiB resident), steps back to back"
           if in_bytes > 2 * L2_BYTES else
@@ -133,7 +138,8 @@ def workload_config(spec, wl, graph: bool) -> dict:
     return {"workload": spec.name, "n_tokens": wl.n_tokens, "d": spec.d, "vocab": spec.vocab,
             "launch": "CUDA graph replay of one step" if graph else "eager",
             "roots": spec.n_roots, "k": spec.k, "conts": int(wl.cont_offsets.numel() - 1),
-            "context_rows_per_step": 2 * wl.n_tokens, "l2": l2}
+            "context_rows_per_step": 2 * wl.n_tokens, "l2": l2,
+            **({"vocab_shards": shards} if shards > 0 else {})}
 
 
 class ClockSampler:
@@ -200,10 +206,24 @@ def clock_suspect(clk) -> bool:
     return not reasons and bool(smax) and clk["sm_mhz"] < 0.8 * smax
 
 
-class Path:
-    """Device buffers and the four library calls of one step."""
+def shard_bounds(vocab: int, shards: int) -> list:
+    """Row boundaries of at most `shards` nearly equal vocabulary shards, cut
+    at multiples of the kernel's 256-row tile (the last shard takes the rest;
+    a vocabulary too small for that many cuts gets fewer shards)."""
+    b = [0]
+    for p in range(1, shards):
+        c = min(vocab, round(p * vocab / shards / 256) * 256)
+        if b[-1] < c < vocab:
+            b.append(c)
+    b.append(vocab)
+    return b
 
-    def __init__(self, hdl, wl):
+
+class Path:
+    """Device buffers and the four library calls of one step (re-scoring
+    through the vocabulary-parallel entry points when `shards` > 0)."""
+
+    def __init__(self, hdl, wl, shards: int = 0):
         self.hdl, self.wl = hdl, wl
         dev = wl.h_orig.device
         N, R, k = wl.n_tokens, wl.n_roots, wl.spec.k
@@ -211,7 +231,14 @@ class Path:
         self.lp0 = torch.empty(N, dtype=torch.float32, device=dev)
         self.lp1 = torch.empty_like(self.lp0)
         self.delta = torch.empty_like(self.lp0)
-        need = hdl.hdl_rescore_workspace_bytes(N, wl.spec.d, wl.spec.vocab, wl.h_orig.dtype)
+        self.bounds = shard_bounds(wl.spec.vocab, shards) if shards > 0 else None
+        if self.bounds is None:
+            need = hdl.hdl_rescore_workspace_bytes(N, wl.spec.d, wl.spec.vocab, wl.h_orig.dtype)
+        else:   # the shards' calls run one after the other on one stream: one workspace
+            need = max(hdl.hdl_rescore_shard_workspace_bytes(N, wl.spec.d, b1 - b0,
+                                                              wl.h_orig.dtype)
+                       for b0, b1 in zip(self.bounds[:-1], self.bounds[1:]))
+            self.stats = torch.empty((shards, 2, N, 4), dtype=torch.float32, device=dev)
         self.ws = torch.empty(need, dtype=torch.uint8, device=dev)
         self.bp = torch.empty((R, k), dtype=torch.int32, device=dev)
         self.ns = torch.empty(R, dtype=torch.int32, device=dev)
@@ -221,8 +248,20 @@ class Path:
 
     def rescore(self, stream):
         w = self.wl
-        self.hdl.hdl_rescore(w.h_orig, w.h_hind, w.w, w.targets, self.lp0, self.lp1,
-                             self.delta, self.ws, stream=stream)
+        if self.bounds is None:
+            self.hdl.hdl_rescore(w.h_orig, w.h_hind, w.w, w.targets, self.lp0, self.lp1,
+                                 self.delta, self.ws, stream=stream)
+            return
+        for p, (b0, b1) in enumerate(zip(self.bounds[:-1], self.bounds[1:])):
+            self.hdl.hdl_rescore_shard(w.h_orig, w.h_hind, w.w[b0:b1], w.targets, b0,
+                                       stats=self.stats[p], workspace=self.ws, stream=stream)
+        self.hdl.hdl_merge_vocab_shards(self.stats, self.lp0, self.lp1, self.delta,
+                                        want_entropy=False, stream=stream)
+
+    def launches_per_step(self) -> int:
+        # re-scoring (sharded: per shard the kernel and its statistics pass,
+        # then the merge), selection, allocation, masks
+        return (1 if self.bounds is None else 2 * (len(self.bounds) - 1) + 1) + 3
 
     def downstream(self, stream):
         w, h = self.wl, self.hdl
@@ -233,7 +272,6 @@ class Path:
                                    stream=stream)
         h.hdl_suffix_mask(self.cb, w.cont_offsets, w.cont_valid, mask=self.mask, stream=stream)
 
-    LAUNCHES_PER_STEP = 4  # rescore (fused GEMM + LSE + merge), select, assign, mask
 
 
 def dist_setup():
@@ -452,7 +490,9 @@ def run_reference(args, world, rank):
             "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": 1e3 * wall / max(1, args.steps), "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-            "config": workload_config(spec, wl, args.graph),
+            "config": workload_config(spec, wl, args.graph,
+                                      len(shard_bounds(spec.vocab, args.shards)) - 1
+                                      if args.shards > 0 else 0),
             "cpu_baseline": cb,
             "e2e": {"value": value, "unit": "root tokens/s", "h2d_bytes_per_step": 0,
                     "d2h_bytes_per_step": 0}}
@@ -469,7 +509,7 @@ def run_gpu(args, world, rank, local):
     dev = torch.device("cuda", local)
     wl = hdl_synth.generate(spec, device=dev)
     torch.cuda.synchronize()
-    path = Path(hdl, wl)
+    path = Path(hdl, wl, args.shards)
     stream = torch.cuda.current_stream()
     N, d, V = wl.n_tokens, spec.d, spec.vocab
     flops = 2.0 * (2 * N) * d * V
@@ -551,7 +591,7 @@ def run_gpu(args, world, rank, local):
                 "cont_offsets", "cont_valid")
         host_in = {k: getattr(wl, k).cpu().pin_memory() for k in keys}
         wl2 = dataclasses.replace(wl, **{k: torch.empty_like(getattr(wl, k)) for k in keys})
-        sets = [(wl, path), (wl2, Path(hdl, wl2))]
+        sets = [(wl, path), (wl2, Path(hdl, wl2, args.shards))]
         host_out = [[torch.empty(t.shape, dtype=t.dtype, pin_memory=True)
                      for t in (p_.bp, p_.ns, p_.bd, p_.mask)] for _, p_ in sets]
         h2d = sum(t.numel() * t.element_size() for t in host_in.values())
@@ -634,9 +674,11 @@ def run_gpu(args, world, rank, local):
         cpu = cpu_oracle_sample(wl, args.cpu_seconds,
                                 gpu_logp=(path.lp0.cpu().numpy(), path.lp1.cpu().numpy()))
 
-    config = workload_config(spec, wl, args.graph)
+    config = workload_config(spec, wl, args.graph,
+                             len(path.bounds) - 1 if path.bounds is not None else 0)
+    launches = path.launches_per_step()
     extra = None
-    if world == 1 and spec.name == "code" and not args.no_extra:
+    if world == 1 and spec.name == "code" and not args.no_extra and args.shards == 0:
         # free the default workload, then the other large ones, one at a time
         del path, wl, flush, graph
         torch.cuda.empty_cache()
@@ -666,14 +708,17 @@ def run_gpu(args, world, rank, local):
         "config": config,
         "tflops": flops * args.steps / (total_ms / 1e3) / 1e12,
         "pct_bf16_peak": 100.0 * (flops * args.steps / (total_ms / 1e3) / 1e12) / burst,
-        "roofline": {"bound": "tensor", "kernel": "rescore_lse_kernel",
+        "roofline": {"bound": "tensor",
+                     "kernel": ("rescore_lse_kernel" if args.shards == 0 else
+                                f"rescore_lse_kernel over {args.shards} vocabulary shards "
+                                "(+ shard statistics and merge)"),
                      "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
                      "frac": achieved / peak, "peak_kind": kind,
                      ("frac_of_burst" if long_run else "frac_of_sustained"): achieved / other,
-                     "traffic": committed_traffic(spec.name),
+                     "traffic": committed_traffic(spec.name) if args.shards == 0 else None,
                      "rescore_ms": rescore_ms},
         "cpu_baseline": cpu, "e2e": e2e, "clocks": clk,
-        "gpu_launches": Path.LAUNCHES_PER_STEP * args.steps,
+        "gpu_launches": launches * args.steps,
     }
     if extra is not None:
         line["workloads"] = extra

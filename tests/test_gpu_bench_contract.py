@@ -78,3 +78,15 @@ def test_graph_replay_line():
     e = d["e2e"]
     assert num(e["value"]) and e["value"] > 0 and "graph" in e["overlap"]
     assert e["h2d_bytes_per_step"] > 0 and e["d2h_bytes_per_step"] > 0
+
+
+def test_vocab_sharded_line():
+    """--shards: re-scoring through hdl_rescore_shard on row shards of W and
+    hdl_merge_vocab_shards on one GPU; the timed steps' log-probs still match
+    the oracle on its sampled tokens."""
+    d = run("--workload", "tiny", "--steps", "3", "--warmup", "3", "--shards", "3",
+            "--cpu-seconds", "1", "--no-e2e")
+    assert d["config"]["vocab_shards"] == 3
+    assert "shards" in d["roofline"]["kernel"] and d["roofline"]["traffic"] is None
+    assert d["cpu_baseline"]["parity"]["within"] is True
+    assert d["gpu_launches"] == 3 * (2 * 3 + 1 + 3)
