@@ -45,6 +45,10 @@ def parse():
                         "(math_f32) gives fp32 hidden states and LM head (tf32 products)")
     p.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
     p.add_argument("--no-e2e", action="store_true")
+    p.add_argument("--entropy", action="store_true",
+                   help="re-score through hdl_rescore_ex with the original context's "
+                        "next-token entropies as a fourth output (the Entropy selector's "
+                        "signal, computed in the same vocabulary walk)")
     p.add_argument("--shards", type=int, default=0,
                    help="re-score through the vocabulary-parallel entry points on this one GPU: "
                         "W cut into this many row shards (at 256-row tile boundaries), one "
@@ -126,10 +130,11 @@ def input_bytes(wl) -> int:
     return sum(t.numel() * t.element_size() for t in (wl.h_orig, wl.h_hind, wl.w))
 
 
-def workload_config(spec, wl, graph: bool, shards: int = 0) -> dict:
+def workload_config(spec, wl, graph: bool, shards: int = 0, entropy: bool = False) -> dict:
     """The ``config`` of the JSON line, identical for both arms: the workload,
     its sizes, how L2 is handled between timed steps and, when the LM head is
-    cut into vocabulary shards, their number."""
+    cut into vocabulary shards, their number, or when the re-scoring also
+    returns next-token entropies, that."""
     in_bytes = input_bytes(wl)
     l2 = (f"inputs larger than L2 ({in_bytes / 2**30:.2f} GiB resident), steps back to back"
           if in_bytes > 2 * L2_BYTES else
@@ -139,7 +144,8 @@ def workload_config(spec, wl, graph: bool, shards: int = 0) -> dict:
             "launch": "CUDA graph replay of one step" if graph else "eager",
             "roots": spec.n_roots, "k": spec.k, "conts": int(wl.cont_offsets.numel() - 1),
             "context_rows_per_step": 2 * wl.n_tokens, "l2": l2,
-            **({"vocab_shards": shards} if shards > 0 else {})}
+            **({"vocab_shards": shards} if shards > 0 else {}),
+            **({"entropy_orig": True} if entropy else {})}
 
 
 class ClockSampler:
@@ -223,8 +229,9 @@ class Path:
     """Device buffers and the four library calls of one step (re-scoring
     through the vocabulary-parallel entry points when `shards` > 0)."""
 
-    def __init__(self, hdl, wl, shards: int = 0):
+    def __init__(self, hdl, wl, shards: int = 0, entropy: bool = False):
         self.hdl, self.wl = hdl, wl
+        self.entropy = entropy
         dev = wl.h_orig.device
         N, R, k = wl.n_tokens, wl.n_roots, wl.spec.k
         self.C = wl.cont_offsets.numel() - 1
@@ -232,7 +239,13 @@ class Path:
         self.lp1 = torch.empty_like(self.lp0)
         self.delta = torch.empty_like(self.lp0)
         self.bounds = shard_bounds(wl.spec.vocab, shards) if shards > 0 else None
-        if self.bounds is None:
+        if entropy:
+            if shards > 0:
+                raise SystemExit("--entropy and --shards are separate measurements")
+            self.ent0 = torch.empty_like(self.lp0)
+            need = hdl.hdl_rescore_ex_workspace_bytes(N, wl.spec.d, wl.spec.vocab,
+                                                      wl.h_orig.dtype, entropy=True)
+        elif self.bounds is None:
             need = hdl.hdl_rescore_workspace_bytes(N, wl.spec.d, wl.spec.vocab, wl.h_orig.dtype)
         else:   # the shards' calls run one after the other on one stream: one workspace
             need = max(hdl.hdl_rescore_shard_workspace_bytes(N, wl.spec.d, b1 - b0,
@@ -248,6 +261,11 @@ class Path:
 
     def rescore(self, stream):
         w = self.wl
+        if self.entropy:
+            self.hdl.hdl_rescore_ex(w.h_orig, w.h_hind, w.w, w.targets, self.lp0, self.lp1,
+                                    self.delta, entropy_orig=self.ent0, workspace=self.ws,
+                                    stream=stream)
+            return
         if self.bounds is None:
             self.hdl.hdl_rescore(w.h_orig, w.h_hind, w.w, w.targets, self.lp0, self.lp1,
                                  self.delta, self.ws, stream=stream)
@@ -492,7 +510,7 @@ def run_reference(args, world, rank):
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
             "config": workload_config(spec, wl, args.graph,
                                       len(shard_bounds(spec.vocab, args.shards)) - 1
-                                      if args.shards > 0 else 0),
+                                      if args.shards > 0 else 0, args.entropy),
             "cpu_baseline": cb,
             "e2e": {"value": value, "unit": "root tokens/s", "h2d_bytes_per_step": 0,
                     "d2h_bytes_per_step": 0}}
@@ -509,7 +527,7 @@ def run_gpu(args, world, rank, local):
     dev = torch.device("cuda", local)
     wl = hdl_synth.generate(spec, device=dev)
     torch.cuda.synchronize()
-    path = Path(hdl, wl, args.shards)
+    path = Path(hdl, wl, args.shards, args.entropy)
     stream = torch.cuda.current_stream()
     N, d, V = wl.n_tokens, spec.d, spec.vocab
     flops = 2.0 * (2 * N) * d * V
@@ -591,7 +609,7 @@ def run_gpu(args, world, rank, local):
                 "cont_offsets", "cont_valid")
         host_in = {k: getattr(wl, k).cpu().pin_memory() for k in keys}
         wl2 = dataclasses.replace(wl, **{k: torch.empty_like(getattr(wl, k)) for k in keys})
-        sets = [(wl, path), (wl2, Path(hdl, wl2, args.shards))]
+        sets = [(wl, path), (wl2, Path(hdl, wl2, args.shards, args.entropy))]
         host_out = [[torch.empty(t.shape, dtype=t.dtype, pin_memory=True)
                      for t in (p_.bp, p_.ns, p_.bd, p_.mask)] for _, p_ in sets]
         h2d = sum(t.numel() * t.element_size() for t in host_in.values())
@@ -675,10 +693,12 @@ def run_gpu(args, world, rank, local):
                                 gpu_logp=(path.lp0.cpu().numpy(), path.lp1.cpu().numpy()))
 
     config = workload_config(spec, wl, args.graph,
-                             len(path.bounds) - 1 if path.bounds is not None else 0)
+                             len(path.bounds) - 1 if path.bounds is not None else 0,
+                             args.entropy)
     launches = path.launches_per_step()
     extra = None
-    if world == 1 and spec.name == "code" and not args.no_extra and args.shards == 0:
+    if (world == 1 and spec.name == "code" and not args.no_extra and args.shards == 0
+            and not args.entropy):
         # free the default workload, then the other large ones, one at a time
         del path, wl, flush, graph
         torch.cuda.empty_cache()
@@ -709,13 +729,15 @@ def run_gpu(args, world, rank, local):
         "tflops": flops * args.steps / (total_ms / 1e3) / 1e12,
         "pct_bf16_peak": 100.0 * (flops * args.steps / (total_ms / 1e3) / 1e12) / burst,
         "roofline": {"bound": "tensor",
-                     "kernel": ("rescore_lse_kernel" if args.shards == 0 else
+                     "kernel": ("rescore_lse_kernel with entropies" if args.entropy else
+                                "rescore_lse_kernel" if args.shards == 0 else
                                 f"rescore_lse_kernel over {args.shards} vocabulary shards "
                                 "(+ shard statistics and merge)"),
                      "achieved": achieved, "peak": peak, "unit": "TFLOP/s",
                      "frac": achieved / peak, "peak_kind": kind,
                      ("frac_of_burst" if long_run else "frac_of_sustained"): achieved / other,
-                     "traffic": committed_traffic(spec.name) if args.shards == 0 else None,
+                     "traffic": (committed_traffic(spec.name)
+                                 if args.shards == 0 and not args.entropy else None),
                      "rescore_ms": rescore_ms},
         "cpu_baseline": cpu, "e2e": e2e, "clocks": clk,
         "gpu_launches": launches * args.steps,

@@ -90,3 +90,15 @@ def test_vocab_sharded_line():
     assert "shards" in d["roofline"]["kernel"] and d["roofline"]["traffic"] is None
     assert d["cpu_baseline"]["parity"]["within"] is True
     assert d["gpu_launches"] == 3 * (2 * 3 + 1 + 3)
+
+
+def test_entropy_line():
+    """--entropy: the re-scoring call also returns the original context's
+    next-token entropies (hdl_rescore_ex); both arms report it in config."""
+    d = run("--workload", "tiny", "--steps", "3", "--warmup", "3", "--entropy",
+            "--cpu-seconds", "1", "--no-e2e")
+    assert d["config"]["entropy_orig"] is True and "entropies" in d["roofline"]["kernel"]
+    assert d["cpu_baseline"]["parity"]["within"] is True
+    b = run("--impl", "reference", "--workload", "tiny", "--steps", "1", "--warmup", "1",
+            "--entropy")
+    assert b["config"] == d["config"]
