@@ -53,7 +53,7 @@ constexpr int kRowBytes = 128;       // K bytes per stage (one 128-byte swizzle 
 constexpr int kMaxTilesPerChunk = 16;  // up to 4096 vocabulary entries per unit
 constexpr int64_t kMinUnits = 1216;     // 8 x 152: chunks shrink until this many units
 constexpr double kL2Budget = 70e6;      // bytes of L2 the running units' tiles may use
-constexpr int kPairsInFlight = 76;      // CTA pairs resident on 152 SMs
+constexpr int kUnitsInFlight = 152;    // work units running at once: one per SM
 #ifndef HDL_GROUP_M
 #define HDL_GROUP_M 32
 #endif
@@ -103,7 +103,7 @@ struct RescoreArgs {
   int32_t num_vt;      // vocabulary tiles
   int32_t num_chunks;
   int32_t tiles_per_chunk;
-  int32_t num_units;   // work units (per cluster in the cluster modes)
+  int32_t num_units;   // work units (per cluster in the pair mode)
   int32_t group_m;     // M-tiles per rasterisation group (even)
   int32_t target_offset;  // targets are shifted by this (vocabulary shards)
   uint32_t inject;     // test hook: bit 0 = the producer issues no copies
@@ -617,8 +617,8 @@ Geometry geometry(int64_t n, int32_t d, int32_t vocab, hdl_dtype dt) {
   // The chunk: the largest power of two (<= 16 tiles) for which the tiles the
   // concurrently running units touch stay within kL2Budget of the 126 MB L2
   // -- the H tiles of one rasterisation group (group_m x 128 rows) plus the W
-  // tiles of the chunks in flight (one chunk per group_m / 2 running CTA
-  // pairs' worth of units, 76 pairs' worth on 152 SMs).  Past that, W tiles
+  // tiles of the chunks in flight (one chunk per group_m running units, 152
+  // units running at once on 152 SMs).  Past that, W tiles
   // are evicted before the group's last units use them: on the code-shaped
   // workload 4-tile chunks (64 MB) read 90 GB from DRAM per launch instead of
   // 156 GB and run 2.5 % faster than 16-tile ones, agent-shaped (d = 5120)
@@ -628,7 +628,7 @@ Geometry geometry(int64_t n, int32_t d, int32_t vocab, hdl_dtype dt) {
   const double row = static_cast<double>(d) * g.esize;
   const int gm = rescore_group_m();
   const double h_bytes = gm * static_cast<double>(kBM) * row;
-  const double chunks_in_flight = 2.0 * kPairsInFlight / gm;
+  const double chunks_in_flight = static_cast<double>(kUnitsInFlight) / gm;
   g.tiles_per_chunk = kMaxTilesPerChunk;
   while (g.tiles_per_chunk > 1 &&
          h_bytes + chunks_in_flight * g.tiles_per_chunk * kBN * row > kL2Budget)
@@ -707,7 +707,7 @@ bool make_operand_map(CUtensorMap* m, const void* ptr, int64_t rows, int32_t d, 
   return r == CUDA_SUCCESS;
 }
 
-// One persistent CTA per SM (cluster modes: as many clusters of two as can
+// One persistent CTA per SM (pair mode: as many clusters of two as can
 // be resident at once).
 template <bool kTf32, int M, bool kEnt>
 hdl_status launch_rescore(const CUtensorMap& tm_h0, const CUtensorMap& tm_h1,
