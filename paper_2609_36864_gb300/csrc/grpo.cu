@@ -397,11 +397,12 @@ extern "C" hdl_status hdl_grpo_loss(const float* logp_new, const float* logp_old
   int blocks = static_cast<int>(want < cap ? want : cap);
   if (blocks > kMaxBlocks) blocks = kMaxBlocks;
   if (blocks < 1) blocks = 1;
-  // pass 0 sized by its own work: 16 KiB of mask or 8 groups per block
+  // pass 0 sized by its own work: 16 KiB of mask or 8 groups per block, up
+  // to 8 blocks per SM (16384 x 4096 tokens: 14.0 us against 16.7 at 4)
   want = ceil_div(n_tokens, int64_t{16384});
   const int64_t gwant = ceil_div(n_groups, kThreads / 32);
   if (gwant > want) want = gwant;
-  int prep = static_cast<int>(want < 4 * sms ? want : 4 * sms);
+  int prep = static_cast<int>(want < 8 * sms ? want : 8 * sms);
   if (prep > kMaxBlocks) prep = kMaxBlocks;
   if (prep < 1) prep = 1;
   // the denominator counts the mask over [0, n_tokens); the token pass
